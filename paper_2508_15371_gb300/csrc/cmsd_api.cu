@@ -1,0 +1,450 @@
+// C ABI of libcmsd.so: argument checks, workspace layout, launches, timing.
+// The operations are specified in include/cmsd.h.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <map>
+#include <mutex>
+#include <tuple>
+#include <vector>
+
+#include "cmsd.h"
+#include "cmsd_internal.h"
+#include "cmsd_philox.cuh"
+
+using namespace cmsd;
+
+namespace {
+
+thread_local int g_last_cuda = 0;
+
+int cuda_fail(cudaError_t e) {
+  g_last_cuda = (int)e;
+  return CMSD_ECUDA;
+}
+
+std::mutex g_mu;
+std::map<int, int> g_sms;                                   // device -> SM count
+std::map<std::tuple<int, int, int, int, int>, int> g_occ;   // (dev, dtype, mode, sampled, smem) -> blocks/SM
+std::map<std::pair<int, int>, int> g_occ_res;               // (dev, dtype) -> blocks/SM
+
+int device_sms(int* sms) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  std::lock_guard<std::mutex> lk(g_mu);
+  auto it = g_sms.find(dev);
+  if (it == g_sms.end()) {
+    int n = 0;
+    e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e);
+    it = g_sms.emplace(dev, n).first;
+  }
+  *sms = it->second;
+  return CMSD_OK;
+}
+
+int stream_grid(int dtype, int mode, bool sampled, size_t smem, int* grid) {
+  int sms = 0;
+  int rc = device_sms(&sms);
+  if (rc) return rc;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const auto key = std::make_tuple(dev, dtype, mode, sampled ? 1 : 0, (int)smem);
+  std::lock_guard<std::mutex> lk(g_mu);
+  auto it = g_occ.find(key);
+  if (it == g_occ.end()) {
+    int nb = 0;
+    cudaError_t e = occupancy_stream(dtype, mode, sampled, smem, &nb);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (nb < 1) nb = 1;
+    it = g_occ.emplace(key, nb).first;
+  }
+  *grid = sms * it->second;
+  return CMSD_OK;
+}
+
+int resample_grid(int dtype, int* grid) {
+  int sms = 0;
+  int rc = device_sms(&sms);
+  if (rc) return rc;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lk(g_mu);
+  auto key = std::make_pair(dev, dtype);
+  auto it = g_occ_res.find(key);
+  if (it == g_occ_res.end()) {
+    int nb = 0;
+    cudaError_t e = occupancy_resample(dtype, &nb);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (nb < 1) nb = 1;
+    it = g_occ_res.emplace(key, nb).first;
+  }
+  *grid = sms * it->second;
+  return CMSD_OK;
+}
+
+// ---------------------------------------------------------------- workspace
+
+constexpr size_t kAlign = 256;
+size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+struct Layout {
+  size_t err, row_done, seq_done, res_done, rej_count, res_cta_done;
+  size_t rej_list, seq_n, row_conf, row_acc, row_targmax, row_dstat, row_tstat, part, rpart;
+  size_t total;
+};
+
+// The error word sits at offset 0 so that cmsd_workspace_errors needs no sizes.
+Layout make_layout(int B, int K, int wmax) {
+  Layout L;
+  const size_t BK = (size_t)B * (size_t)K;
+  size_t o = 0;
+  L.err = o; o += up(sizeof(unsigned));
+  L.row_done = o; o += up(BK * sizeof(int));
+  L.seq_done = o; o += up((size_t)B * sizeof(int));
+  L.res_done = o; o += up((size_t)B * sizeof(int));
+  L.rej_count = o; o += up(sizeof(int));
+  L.res_cta_done = o; o += up(sizeof(int));
+  L.rej_list = o; o += up((size_t)B * sizeof(int));
+  L.seq_n = o; o += up((size_t)B * sizeof(int));
+  L.row_conf = o; o += up(BK * sizeof(float));
+  L.row_acc = o; o += up(BK * sizeof(int));
+  L.row_targmax = o; o += up(BK * sizeof(int));
+  L.row_dstat = o; o += up(BK * sizeof(float2));
+  L.row_tstat = o; o += up(BK * sizeof(float2));
+  L.part = o; o += up((BK + (size_t)wmax) * sizeof(Partial));
+  L.rpart = o; o += up(((size_t)B + (size_t)wmax) * sizeof(RacePartial));
+  L.total = o;
+  return L;
+}
+
+Workspace carve(void* ws, const Layout& L) {
+  char* p = (char*)ws;
+  Workspace W;
+  W.err = (unsigned*)(p + L.err);
+  W.row_done = (int*)(p + L.row_done);
+  W.seq_done = (int*)(p + L.seq_done);
+  W.res_done = (int*)(p + L.res_done);
+  W.rej_count = (int*)(p + L.rej_count);
+  W.res_cta_done = (int*)(p + L.res_cta_done);
+  W.rej_list = (int*)(p + L.rej_list);
+  W.seq_n = (int*)(p + L.seq_n);
+  W.row_conf = (float*)(p + L.row_conf);
+  W.row_acc = (int*)(p + L.row_acc);
+  W.row_targmax = (int*)(p + L.row_targmax);
+  W.row_dstat = (float2*)(p + L.row_dstat);
+  W.row_tstat = (float2*)(p + L.row_tstat);
+  W.part = (Partial*)(p + L.part);
+  W.rpart = (RacePartial*)(p + L.rpart);
+  return W;
+}
+
+int wmax_warps(int* wmax) {
+  int sms = 0;
+  int rc = device_sms(&sms);
+  if (rc) return rc;
+  *wmax = sms * kMaxWarpsPerSM;
+  return CMSD_OK;
+}
+
+// ---------------------------------------------------------------- timing
+
+struct Profiler {
+  bool on = false;
+  int max_calls = 0;
+  int n = 0;
+  std::vector<cudaEvent_t> ev;   // 3 per call: start, after stream kernel, after resample
+} g_prof;
+
+void prof_record(int slot, cudaStream_t s) {
+  if (!g_prof.on || g_prof.n >= g_prof.max_calls) return;
+  cudaEventRecord(g_prof.ev[3 * g_prof.n + slot], s);
+  if (slot == 2) ++g_prof.n;
+}
+
+// ---------------------------------------------------------------- checks
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+int check_sizes(int B, int K, int V, int dtype, const int32_t* k_row) {
+  if (dtype != CMSD_F32 && dtype != CMSD_BF16) return CMSD_EDTYPE;
+  if (B < 0 || K < 0 || K > 1024 || V < 2) return CMSD_EINVAL;
+  if ((long long)B * (long long)K > 0x7FFFFFFFLL) return CMSD_EINVAL;
+  if ((double)B * (double)K * (double)V >= 70368744177664.0) return CMSD_EINVAL;   // 2^46
+  if (k_row && B > kMaxRaggedB) return CMSD_EINVAL;
+  return CMSD_OK;
+}
+
+int check_params(const cmsd_params* p, bool need_rule) {
+  if (!p) return CMSD_EINVAL;
+  if (need_rule && p->rule != CMSD_RULE_PAPER && p->rule != CMSD_RULE_SAMPLED) return CMSD_EDTYPE;
+  if (p->k_min < 1 || p->k_max < p->k_min) return CMSD_EINVAL;
+  float sum = 0.f;
+  for (int j = 0; j < 3; ++j) {
+    if (!(p->lambda[j] >= 0.f && p->lambda[j] <= 1.f)) return CMSD_EINVAL;
+    sum += p->lambda[j];
+  }
+  if (fabsf(sum - 1.0f) > 1e-5f) return CMSD_EINVAL;
+  if (!(p->beta_sig > 0.f) || !isfinite(p->beta_sig)) return CMSD_EINVAL;
+  if (p->beta_rank < 0) return CMSD_EINVAL;
+  if (!(p->alpha > 0.f && p->alpha <= 1.f)) return CMSD_EINVAL;
+  if (!isfinite(p->tau_base) || !isfinite(p->gamma)) return CMSD_EINVAL;
+  if (p->tau_sign != 1 && p->tau_sign != -1) return CMSD_EINVAL;
+  return CMSD_OK;
+}
+
+void fill_params(StreamArgs& a, const cmsd_params* p) {
+  a.k_min = p->k_min;
+  a.k_max = p->k_max;
+  a.lam0 = p->lambda[0];
+  a.lam1 = p->lambda[1];
+  a.lam2 = p->lambda[2];
+  a.beta_sig = p->beta_sig;
+  a.beta_rank = p->beta_rank;
+  a.alpha = p->alpha;
+  a.tau_base = p->tau_base;
+  a.gamma = p->gamma;
+  a.tau_sign = p->tau_sign;
+}
+
+int launch(int dtype, int mode, bool sampled, StreamArgs& a, void* ws, size_t ws_bytes,
+           cudaStream_t s) {
+  int wmax = 0;
+  int rc = wmax_warps(&wmax);
+  if (rc) return rc;
+  const Layout L = make_layout(a.B, a.K, wmax);
+  if (!ws || ws_bytes < L.total) return CMSD_ENOWS;
+  a.ws = carve(ws, L);
+  const size_t smem = a.k_row ? (size_t)(a.B + 1) * sizeof(int) : 0;
+  int grid = 0;
+  rc = stream_grid(dtype, mode, sampled, smem, &grid);
+  if (rc) return rc;
+  a.nwarps = grid * kWarpsPerBlock;
+  prof_record(0, s);
+  cudaError_t e = dtype == CMSD_F32 ? launch_stream_f32(mode, sampled, a, grid, smem, s)
+                                    : launch_stream_bf16(mode, sampled, a, grid, smem, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  prof_record(1, s);
+  if (sampled && mode != kModeConf) {
+    int g2 = 0;
+    rc = resample_grid(dtype, &g2);
+    if (rc) return rc;
+    StreamArgs b = a;
+    b.nwarps = g2 * kWarpsPerBlock;
+    e = dtype == CMSD_F32 ? launch_resample_f32(b, g2, s) : launch_resample_bf16(b, g2, s);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
+  prof_record(2, s);
+  return CMSD_OK;
+}
+
+StreamArgs blank_args() {
+  StreamArgs a;
+  memset(&a, 0, sizeof(a));
+  return a;
+}
+
+}  // namespace
+
+// ============================================================ C ABI
+
+extern "C" {
+
+void cmsd_params_default(cmsd_params* p, int K, int rule) {
+  if (!p) return;
+  p->k_min = 1;
+  p->k_max = K > 0 ? K : 1;
+  p->lambda[0] = p->lambda[1] = p->lambda[2] = 1.0f / 3.0f;
+  p->beta_sig = 1.0f;
+  p->beta_rank = rule == CMSD_RULE_SAMPLED ? 0 : 3;
+  p->alpha = 1.0f;
+  p->tau_base = 0.1f;
+  p->gamma = 1.0f;
+  p->tau_sign = 1;
+  p->rule = rule;
+}
+
+size_t cmsd_workspace_bytes(int B, int K, int V) {
+  (void)V;
+  if (B < 0 || K < 0) return 0;
+  int wmax = 0;
+  if (wmax_warps(&wmax)) return 0;
+  return make_layout(B, K, wmax).total;
+}
+
+int cmsd_workspace_init(void* ws, size_t ws_bytes, void* stream) {
+  if (!ws || ws_bytes == 0) return CMSD_ENOWS;
+  cudaError_t e = cudaMemsetAsync(ws, 0, ws_bytes, (cudaStream_t)stream);
+  return e == cudaSuccess ? CMSD_OK : cuda_fail(e);
+}
+
+int cmsd_workspace_errors(void* ws, size_t ws_bytes, void* stream, uint32_t* flags_out) {
+  if (!ws || ws_bytes < sizeof(unsigned) || !flags_out) return CMSD_EINVAL;
+  unsigned h = 0;
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = cudaMemcpyAsync(&h, ws, sizeof(unsigned), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ws, 0, sizeof(unsigned), s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  *flags_out = h;
+  return CMSD_OK;
+}
+
+int cmsd_confidence(const void* draft_logits, int B, int K, int V, int dtype, const int32_t* k_row,
+                    const cmsd_params* p, float* H, float* margin, int32_t* argmax, float* conf,
+                    float* lse, int32_t* k_next, void* ws, size_t ws_bytes, void* stream) {
+  int rc = check_sizes(B, K, V, dtype, k_row);
+  if (rc) return rc;
+  rc = check_params(p, false);
+  if (rc) return rc;
+  if (B == 0 || K == 0) return CMSD_OK;
+  if (!draft_logits) return CMSD_EINVAL;
+  if (!aligned16(draft_logits)) return CMSD_EALIGN;
+  StreamArgs a = blank_args();
+  a.draft = draft_logits;
+  a.k_row = k_row;
+  a.B = B; a.K = K; a.V = V;
+  fill_params(a, p);
+  a.H = H; a.margin = margin; a.argmax = argmax; a.conf = conf; a.lse = lse; a.k_next = k_next;
+  return launch(dtype, kModeConf, false, a, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+int cmsd_verify(const void* draft_logits, const void* target_logits, const int32_t* draft_tokens,
+                const int32_t* k_row, int B, int K, int V, int dtype, const cmsd_params* p,
+                const float* conf, const float* draft_lse, uint64_t seed, uint32_t iteration,
+                int32_t* n_accept, int32_t* out_tokens, uint8_t* accept, void* ws, size_t ws_bytes,
+                void* stream) {
+  int rc = check_sizes(B, K, V, dtype, k_row);
+  if (rc) return rc;
+  rc = check_params(p, true);
+  if (rc) return rc;
+  if (B == 0 || K == 0) return CMSD_OK;
+  const bool sampled = p->rule == CMSD_RULE_SAMPLED;
+  if (!draft_logits || !target_logits || !draft_tokens || !conf || !n_accept || !out_tokens)
+    return CMSD_EINVAL;
+  if (sampled && !draft_lse) return CMSD_EINVAL;
+  if (!aligned16(draft_logits) || !aligned16(target_logits)) return CMSD_EALIGN;
+  StreamArgs a = blank_args();
+  a.draft = draft_logits;
+  a.target = target_logits;
+  a.tokens = draft_tokens;
+  a.k_row = k_row;
+  a.B = B; a.K = K; a.V = V;
+  fill_params(a, p);
+  a.seed = seed;
+  a.iteration = iteration;
+  a.conf_in = conf;
+  a.lse_in = draft_lse;
+  a.n_accept = n_accept; a.out_tokens = out_tokens; a.accept = accept;
+  return launch(dtype, kModeVerify, sampled, a, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+int cmsd_confidence_verify(const void* draft_logits, const void* target_logits,
+                           const int32_t* draft_tokens, const int32_t* k_row, int B, int K, int V,
+                           int dtype, const cmsd_params* p, uint64_t seed, uint32_t iteration,
+                           float* H, float* margin, int32_t* argmax, float* conf, float* lse,
+                           int32_t* k_next, int32_t* n_accept, int32_t* out_tokens, uint8_t* accept,
+                           void* ws, size_t ws_bytes, void* stream) {
+  int rc = check_sizes(B, K, V, dtype, k_row);
+  if (rc) return rc;
+  rc = check_params(p, true);
+  if (rc) return rc;
+  if (B == 0 || K == 0) return CMSD_OK;
+  if (!draft_logits || !target_logits || !draft_tokens || !n_accept || !out_tokens) return CMSD_EINVAL;
+  if (!aligned16(draft_logits) || !aligned16(target_logits)) return CMSD_EALIGN;
+  const bool sampled = p->rule == CMSD_RULE_SAMPLED;
+  StreamArgs a = blank_args();
+  a.draft = draft_logits;
+  a.target = target_logits;
+  a.tokens = draft_tokens;
+  a.k_row = k_row;
+  a.B = B; a.K = K; a.V = V;
+  fill_params(a, p);
+  a.seed = seed;
+  a.iteration = iteration;
+  a.H = H; a.margin = margin; a.argmax = argmax; a.conf = conf; a.lse = lse; a.k_next = k_next;
+  a.n_accept = n_accept; a.out_tokens = out_tokens; a.accept = accept;
+  return launch(dtype, kModeFused, sampled, a, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+uint32_t cmsd_philox_u32(uint64_t seed, uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3, int word) {
+  const U4 w = philox4x32_10(U4{c0, c1, c2, c3}, seed_lo(seed), seed_hi(seed));
+  switch (word & 3) {
+    case 0: return w.x;
+    case 1: return w.y;
+    case 2: return w.z;
+    default: return w.w;
+  }
+}
+
+int cmsd_philox_fill(uint64_t seed, uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3, uint32_t* out,
+                     size_t n, void* stream) {
+  if (n == 0) return CMSD_OK;
+  if (!out) return CMSD_EINVAL;
+  cudaError_t e = launch_philox_fill(seed, c0, c1, c2, c3, out, n, (cudaStream_t)stream);
+  return e == cudaSuccess ? CMSD_OK : cuda_fail(e);
+}
+
+int cmsd_profile_start(int max_calls) {
+  if (max_calls < 0) return CMSD_EINVAL;
+  const size_t need = (size_t)max_calls * 3;
+  while (g_prof.ev.size() < need) {
+    cudaEvent_t e;
+    cudaError_t err = cudaEventCreate(&e);
+    if (err != cudaSuccess) return cuda_fail(err);
+    g_prof.ev.push_back(e);
+  }
+  g_prof.on = true;
+  g_prof.max_calls = max_calls;
+  g_prof.n = 0;
+  return CMSD_OK;
+}
+
+int cmsd_profile_stop(float* stream_ms, float* resample_ms, int max_out, int* n_out) {
+  g_prof.on = false;
+  const int n = g_prof.n < max_out ? g_prof.n : max_out;
+  for (int j = 0; j < n; ++j) {
+    cudaError_t e = cudaEventSynchronize(g_prof.ev[3 * j + 2]);
+    if (e != cudaSuccess) return cuda_fail(e);
+    float a = 0.f, b = 0.f;
+    e = cudaEventElapsedTime(&a, g_prof.ev[3 * j], g_prof.ev[3 * j + 1]);
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&b, g_prof.ev[3 * j + 1], g_prof.ev[3 * j + 2]);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (stream_ms) stream_ms[j] = a;
+    if (resample_ms) resample_ms[j] = b;
+  }
+  if (n_out) *n_out = n;
+  g_prof.n = 0;
+  return CMSD_OK;
+}
+
+int cmsd_launch_info(int dtype, int* warps_out, int* sms_out) {
+  if (dtype != CMSD_F32 && dtype != CMSD_BF16) return CMSD_EDTYPE;
+  int sms = 0, grid = 0;
+  int rc = device_sms(&sms);
+  if (rc) return rc;
+  rc = stream_grid(dtype, kModeFused, true, 0, &grid);
+  if (rc) return rc;
+  if (warps_out) *warps_out = grid * kWarpsPerBlock;
+  if (sms_out) *sms_out = sms;
+  return CMSD_OK;
+}
+
+const char* cmsd_strerror(int code) {
+  switch (code) {
+    case CMSD_OK: return "ok";
+    case CMSD_EINVAL: return "invalid argument";
+    case CMSD_EDTYPE: return "unknown dtype or rule";
+    case CMSD_ECUDA: return "CUDA runtime error";
+    case CMSD_ENOWS: return "workspace missing or too small";
+    case CMSD_EALIGN: return "logit pointer not 16-byte aligned";
+    default: return "unknown error";
+  }
+}
+
+int cmsd_last_cuda_error(void) { return g_last_cuda; }
+
+}  // extern "C"

@@ -1,0 +1,92 @@
+// Device generator of the decode-loop simulation's synthetic logits
+// (include/cmsd_workload.h).  Input generation only: bit-identical to the
+// host recipe (table lookups and IEEE float adds/multiplies with no
+// contraction), so the CPU oracle can regenerate the same rows.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "cmsd_philox.cuh"
+#include "cmsd_workload.h"
+
+namespace {
+
+constexpr uint32_t kGenDNoise = 0xC0000002u;
+constexpr uint32_t kGenTNoise = 0xC0000003u;
+constexpr uint32_t kGenSpike = 0xC0000004u;
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ uint32_t half16(const cmsd::U4& w, int j) {
+  const uint32_t word = (j >> 1) == 0 ? w.x : (j >> 1) == 1 ? w.y : (j >> 1) == 2 ? w.z : w.w;
+  return (j & 1) ? (word >> 16) : (word & 0xFFFFu);
+}
+
+__global__ void __launch_bounds__(kThreads) gen_rows_kernel(const float* __restrict__ table,
+                                                            const float* __restrict__ heights_it,
+                                                            uint32_t it, int B, int K_max, int V,
+                                                            const int32_t* __restrict__ k_row,
+                                                            uint32_t k0, uint32_t k1, float* draft,
+                                                            float* target, int32_t* tokens) {
+  const int row = blockIdx.x;
+  const int b = row / K_max;
+  const int i = row - b * K_max;
+  if (k_row) {
+    int k = k_row[b];
+    k = k < 0 ? 0 : (k > K_max ? K_max : k);
+    if (i >= k) return;
+  }
+  const float h = heights_it[b];
+  const cmsd::U4 sw = cmsd::philox4x32_10(cmsd::U4{0u, (uint32_t)row, it, kGenSpike}, k0, k1);
+  const int spike = (int)(((uint64_t)sw.x * (uint64_t)V) >> 32);
+  float* dz = draft + (size_t)row * V;
+  float* tz = target + (size_t)row * V;
+
+  float best = -__int_as_float(0x7F800000);
+  int bidx = 0x7FFFFFFF;
+  const int ngrp = (V + 7) / 8;
+  for (int g = threadIdx.x; g < ngrp; g += kThreads) {
+    const cmsd::U4 wd = cmsd::philox4x32_10(cmsd::U4{(uint32_t)g, (uint32_t)row, it, kGenDNoise}, k0, k1);
+    const cmsd::U4 wt = cmsd::philox4x32_10(cmsd::U4{(uint32_t)g, (uint32_t)row, it, kGenTNoise}, k0, k1);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int v = 8 * g + j;
+      if (v < V) {
+        float z = table[half16(wd, j)];
+        if (v == spike) z = __fadd_rn(z, h);
+        const float t = __fadd_rn(z, __fmul_rn(0.8f, table[half16(wt, j)]));
+        dz[v] = z;
+        tz[v] = t;
+        if (z > best) { best = z; bidx = v; }
+      }
+    }
+  }
+  // block argmax, lowest index among equal maxima
+  for (int o = 16; o; o >>= 1) {
+    const float ob = __shfl_xor_sync(0xFFFFFFFFu, best, o);
+    const int oi = __shfl_xor_sync(0xFFFFFFFFu, bidx, o);
+    if (ob > best || (ob == best && oi < bidx)) { best = ob; bidx = oi; }
+  }
+  __shared__ float sb[kThreads / 32];
+  __shared__ int si[kThreads / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) { sb[warp] = best; si[warp] = bidx; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int w = 1; w < kThreads / 32; ++w)
+      if (sb[w] > best || (sb[w] == best && si[w] < bidx)) { best = sb[w]; bidx = si[w]; }
+    tokens[row] = bidx;
+  }
+}
+
+}  // namespace
+
+extern "C" int cmsd_gen_decode_rows(const float* table, const float* heights_it, uint32_t it, int B,
+                                    int K_max, int V, const int32_t* k_row, uint64_t seed,
+                                    float* draft, float* target, int32_t* tokens, void* stream) {
+  if (B < 0 || K_max < 1 || V < 2) return -1;
+  if (B == 0) return 0;
+  if (!table || !heights_it || !draft || !target || !tokens) return -1;
+  gen_rows_kernel<<<B * K_max, kThreads, 0, (cudaStream_t)stream>>>(
+      table, heights_it, it, B, K_max, V, k_row, cmsd::seed_lo(seed), cmsd::seed_hi(seed), draft,
+      target, tokens);
+  return cudaGetLastError() == cudaSuccess ? 0 : -3;
+}
