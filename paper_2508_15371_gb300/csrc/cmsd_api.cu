@@ -218,7 +218,7 @@ int launch(int dtype, int mode, bool sampled, StreamArgs& a, void* ws, size_t ws
   const Layout L = make_layout(a.B, a.K, wmax);
   if (!ws || ws_bytes < L.total) return CMSD_ENOWS;
   a.ws = carve(ws, L);
-  const size_t smem = a.k_row ? (size_t)(a.B + 1) * sizeof(int) : 0;
+  const size_t smem = stream_smem_bytes(a.B, a.k_row != nullptr);
   int grid = 0;
   rc = stream_grid(dtype, mode, sampled, smem, &grid);
   if (rc) return rc;
@@ -426,7 +426,7 @@ int cmsd_launch_info(int dtype, int* warps_out, int* sms_out) {
   int sms = 0, grid = 0;
   int rc = device_sms(&sms);
   if (rc) return rc;
-  rc = stream_grid(dtype, kModeFused, true, 0, &grid);
+  rc = stream_grid(dtype, kModeFused, true, stream_smem_bytes(0, false), &grid);
   if (rc) return rc;
   if (warps_out) *warps_out = grid * kWarpsPerBlock;
   if (sms_out) *sms_out = sms;

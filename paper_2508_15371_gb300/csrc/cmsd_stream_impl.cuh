@@ -4,14 +4,15 @@
 // are laid end to end into one stream of rows * V logits per tensor, and the
 // launched warps (a persistent grid: every SM filled to its occupancy) each
 // take an equal contiguous slice of that stream.  A slice crosses at most a
-// few row boundaries; each piece of a row it covers is a "segment".  A warp
-// reads its segments with 128-bit non-caching loads, keeps per-lane running
-// statistics in registers, reduces them across the warp with shuffles and
-// writes one Partial per segment.  Per-row and per-sequence arrival counters
-// (atomics, no waiting) elect the warp that completes a row to merge its
-// partials into the row's results, and the warp that completes a sequence to
-// run the sequence epilogue (first-reject scan, next draft length, output
-// tokens).  Every logit is read from HBM once.
+// few row boundaries; each piece of a row it covers is a "segment".
+//
+// Memory pipeline.  Each warp owns a ring of kStages shared-memory stages; a
+// stage holds a 1 KB chunk of the drafter row and the matching 1 KB of the
+// target row, filled by bulk copies (cp.async.bulk, TMA) that complete on the
+// stage's mbarrier.  Lane 0 keeps kStages chunks in flight ahead of the warp,
+// across segment boundaries; the warp reads each landed chunk with 128-bit
+// shared loads.  The unaligned head and tail of a segment (fewer than 16
+// bytes each) are read directly from global memory.
 //
 // Per-element work (online softmax, Sec. III.B(1)): with running maximum m,
 //   s  = sum e^(z - m)
@@ -20,54 +21,29 @@
 // grows to m', s and t2 are rescaled by e^(m - m') (t2 also shifted by
 // s * (m - m') log2 e).  The exponent is evaluated as ex2(z*log2e - m*log2e)
 // with the product m*log2e rounded once and shared by every term of the
-// row, so that rounding cancels in p = e^(z-m)/s.
+// row, so that rounding cancels in p = e^(z-m)/s.  Pairs of elements go
+// through the packed f32x2 FMA/ADD pipes.  The target row keeps its maximum,
+// lowest argmax, the count of logits above the drafted token's (saturating at
+// beta_rank) and, for the sampled rule, its own sum of e^(z - m).
 //
-// -inf logits (masked vocabulary) are clamped to kNegClamp before the
-// drafter arithmetic so that e^(z-m) * (z-m) is 0, not NaN.
+// Reduction.  At the end of a segment the warp merges its lanes with
+// shuffles and writes one Partial.  Per-row and per-sequence arrival
+// counters (atomics, no waiting on other warps) elect the warp that completes
+// a row to merge its partials into the row's results, and the warp that
+// completes a sequence to run the sequence epilogue (first-reject scan, next
+// draft length, output tokens).  Every logit is read from HBM once.
+//
+// -inf logits (masked vocabulary) are clamped to -2^100 before the drafter
+// arithmetic so that e^(z-m) * (z-m) is 0, not NaN.
 #pragma once
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "cmsd_device.cuh"
 #include "cmsd_internal.h"
 #include "cmsd_philox.cuh"
 
 namespace cmsd {
-
-constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kLn2 = 0.6931471805599453f;
-constexpr uint32_t kNegClampBits = 0xF14A0000u;       // bf16 value nearest -1e30
-constexpr uint32_t kNegClamp2 = 0xF14AF14Au;          // the same, two bf16 lanes
-constexpr uint32_t kNegInf2 = 0xFF80FF80u;            // -inf, two bf16 lanes
-constexpr float kNegInit = -2.0e30f;                  // below every clamped logit
-constexpr unsigned kFull = 0xFFFFFFFFu;
-
-__device__ __forceinline__ float neg_clamp() { return __uint_as_float(kNegClampBits); }
-
-__device__ __forceinline__ float ex2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-__device__ __forceinline__ uint32_t bmin2(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("min.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-
-__device__ __forceinline__ uint4 ld_stream(const void* p) {
-  uint4 r;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-               : "l"(p));
-  return r;
-}
 
 template <typename T> struct Elem;
 template <> struct Elem<float> {
@@ -84,155 +60,218 @@ template <> struct Elem<uint16_t> {
 // ---------------------------------------------------------------------------
 // per-lane running state
 // ---------------------------------------------------------------------------
+//
+// Each lane walks its elements in increasing index order and keeps, without
+// branches: the exact running maximum and the first vector (or single
+// element) in which it was reached; the exact index inside that vector is
+// resolved at the end of the segment by the lane(s) holding the segment
+// maximum, so the lowest index among equal maxima survives.  The exponent
+// reference `ref` of the sums moves only when the maximum has grown more
+// than kRefSlack above it (rare), so every term is e^(z - ref) <= e^kRefSlack
+// and the final shift to the exact maximum loses no precision.
+
+constexpr float kRefSlack = 4.0f;   // nats
+
+#ifndef CMSD_DRAFT_PACKED
+#define CMSD_DRAFT_PACKED 1
+#endif
+#ifndef CMSD_TARGET_PACKED
+#define CMSD_TARGET_PACKED 1
+#endif
 
 struct DLane {               // drafter
-  float m, negmL;            // running max and -(m*log2e)
-  float s0, s1, t0, t1;      // two interleaved accumulators for ILP
+  float m;                   // exact running max (of clamped logits)
+  float ref;                 // exponent reference of s and t
+  u64 negrL;                 // -(ref*log2e) in both halves
+  u64 s, t;                  // packed (even, odd) sums of e and of e*x, relative to ref
   float f1, f2;              // top-2 of elements taken one at a time (all f32 data)
   uint32_t T1, T2;           // top-2 of bf16 vector elements, per half-word lane
   int pos, posw;             // first unit (start, width) that reached m
 };
 
 struct TLane {               // target
-  float M, negML;
-  float s0, s1;
+  float M;                   // exact running max
+  float ref;
+  u64 negrL;
+  u64 s;                     // packed partial sums of e^(z - ref)
+  float thr;                 // PAPER rule: elements above thr may be counted
   int pos, posw;
   int cnt;
 };
 
 __device__ __forceinline__ void dlane_init(DLane& d) {
   d.m = kNegInit;
-  d.negmL = -(kNegInit * kLog2e);
-  d.s0 = d.s1 = d.t0 = d.t1 = 0.f;
+  d.ref = kNegInit;
+  d.negrL = dup2(-mlog2e(kNegInit));
+  d.s = d.t = 0ull;
   d.f1 = d.f2 = kNegInit;
   d.T1 = d.T2 = kNegInf2;
-  d.pos = 0x7FFFFFFF;
+  d.pos = kIntMax;
   d.posw = 0;
 }
-__device__ __forceinline__ void tlane_init(TLane& t) {
+__device__ __forceinline__ void tlane_init(TLane& t, float c, int beta) {
   t.M = kNegInit;
-  t.negML = -(kNegInit * kLog2e);
-  t.s0 = t.s1 = 0.f;
-  t.pos = 0x7FFFFFFF;
+  t.ref = kNegInit;
+  t.negrL = dup2(-mlog2e(kNegInit));
+  t.s = 0ull;
+  t.pos = kIntMax;
   t.posw = 0;
   t.cnt = 0;
+  t.thr = beta > 0 ? c : pos_inf();
 }
 
-__device__ __forceinline__ void d_raise(DLane& d, float mx, int pos, int posw) {
-  const float nmL = mx * kLog2e;
-  const float dd = -d.negmL - nmL;            // (m_old - m_new) log2e <= 0
-  const float sc = ex2(dd);
-  d.t0 = sc * fmaf(d.s0, dd, d.t0);
-  d.t1 = sc * fmaf(d.s1, dd, d.t1);
-  d.s0 *= sc;
-  d.s1 *= sc;
-  d.m = mx;
-  d.negmL = -nmL;
-  d.pos = pos;
-  d.posw = posw;
+// move the exponent reference up to mx: s *= e^(ref - mx), t likewise
+// (shifted by s * (ref - mx) log2e)
+__device__ __forceinline__ void d_reref(DLane& d, float mx) {
+  const float nrL = mlog2e(mx);
+  const float dd = __fsub_rn(-lo32f(d.negrL), nrL);    // (ref_old - ref_new) log2e <= 0
+  const u64 sc = dup2(ex2(dd));
+  d.t = mul2(sc, fma2(d.s, dup2(dd), d.t));
+  d.s = mul2(d.s, sc);
+  d.ref = mx;
+  d.negrL = dup2(-nrL);
 }
-__device__ __forceinline__ void d_acc0(DLane& d, float z) {
-  const float x = fmaf(z, kLog2e, d.negmL);
-  const float e = ex2(x);
-  d.s0 += e;
-  d.t0 = fmaf(e, x, d.t0);
-}
-__device__ __forceinline__ void d_acc1(DLane& d, float z) {
-  const float x = fmaf(z, kLog2e, d.negmL);
-  const float e = ex2(x);
-  d.s1 += e;
-  d.t1 = fmaf(e, x, d.t1);
+__device__ __forceinline__ void t_reref(TLane& t, float mx) {
+  const float nrL = mlog2e(mx);
+  t.s = mul2(t.s, dup2(ex2(__fsub_rn(-lo32f(t.negrL), nrL))));
+  t.ref = mx;
+  t.negrL = dup2(-nrL);
 }
 
-__device__ __forceinline__ void t_raise(TLane& t, float mx, int pos, int posw, bool sampled) {
-  const float nmL = mx * kLog2e;
-  if (sampled) {
-    const float sc = ex2(-t.negML - nmL);
-    t.s0 *= sc;
-    t.s1 *= sc;
-  }
-  t.M = mx;
-  t.negML = -nmL;
-  t.pos = pos;
-  t.posw = posw;
+// accumulate a pair of (clamped) drafter logits given as packed floats
+__device__ __forceinline__ void d_acc(DLane& d, u64 z) {
+#if CMSD_DRAFT_PACKED
+  const u64 x = fma2(z, dup2(kLog2e), d.negrL);
+  const u64 e = ex2_2(x);
+  d.s = add2(d.s, e);
+  d.t = fma2(e, x, d.t);
+#else
+  const float nr = lo32f(d.negrL);
+  const float xa = fmaf(lo32f(z), kLog2e, nr), xb = fmaf(hi32f(z), kLog2e, nr);
+  const float ea = ex2(xa), eb = ex2(xb);
+  d.s = pack2(lo32f(d.s) + ea, hi32f(d.s) + eb);
+  d.t = pack2(fmaf(ea, xa, lo32f(d.t)), fmaf(eb, xb, hi32f(d.t)));
+#endif
+}
+__device__ __forceinline__ void t_acc(TLane& t, u64 z) {
+#if CMSD_TARGET_PACKED
+  t.s = add2(t.s, ex2_2(fma2(z, dup2(kLog2e), t.negrL)));
+#else
+  const float nr = lo32f(t.negrL);
+  t.s = pack2(lo32f(t.s) + ex2(fmaf(lo32f(z), kLog2e, nr)), hi32f(t.s) + ex2(fmaf(hi32f(z), kLog2e, nr)));
+#endif
 }
 
-// --- drafter: one element at a time (head/tail, or every f32 element) -------
+// --- drafter: one element at a time (segment heads/tails) --------------------
 __device__ __forceinline__ void d_scalar(DLane& d, float z, int v) {
   z = fmaxf(z, neg_clamp());
   d.f2 = fmaxf(d.f2, fminf(d.f1, z));
   d.f1 = fmaxf(d.f1, z);
-  if (z > d.m) d_raise(d, z, v, 1);
-  d_acc0(d, z);
+  if (z > d.m) { d.pos = v; d.posw = 1; }
+  d.m = fmaxf(d.m, z);
+  if (z > d.ref + kRefSlack) d_reref(d, z);
+  d_acc(d, pack2(z, kNegInit));          // the second half adds e = 0
 }
 
 // --- drafter: 8 bf16 ---------------------------------------------------------
 __device__ __forceinline__ void d_vec(DLane& d, uint4 q, int v) {
-  const uint32_t w0 = bmax2(q.x, kNegClamp2), w1 = bmax2(q.y, kNegClamp2);
-  const uint32_t w2 = bmax2(q.z, kNegClamp2), w3 = bmax2(q.w, kNegClamp2);
-  d.T2 = bmax2(d.T2, bmin2(d.T1, w0)); d.T1 = bmax2(d.T1, w0);
-  d.T2 = bmax2(d.T2, bmin2(d.T1, w1)); d.T1 = bmax2(d.T1, w1);
-  d.T2 = bmax2(d.T2, bmin2(d.T1, w2)); d.T1 = bmax2(d.T1, w2);
-  d.T2 = bmax2(d.T2, bmin2(d.T1, w3)); d.T1 = bmax2(d.T1, w3);
+  const uint32_t w[4] = {bmax2(q.x, kNegClamp2), bmax2(q.y, kNegClamp2), bmax2(q.z, kNegClamp2),
+                         bmax2(q.w, kNegClamp2)};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    d.T2 = bmax2(d.T2, bmin2(d.T1, w[k]));
+    d.T1 = bmax2(d.T1, w[k]);
+  }
   const float mx = fmaxf(bf_lo(d.T1), bf_hi(d.T1));
-  if (mx > d.m) d_raise(d, mx, v, 8);
-  d_acc0(d, bf_lo(w0)); d_acc1(d, bf_hi(w0));
-  d_acc0(d, bf_lo(w1)); d_acc1(d, bf_hi(w1));
-  d_acc0(d, bf_lo(w2)); d_acc1(d, bf_hi(w2));
-  d_acc0(d, bf_lo(w3)); d_acc1(d, bf_hi(w3));
+  const bool up = mx > d.m;
+  d.pos = up ? v : d.pos;
+  d.posw = up ? 8 : d.posw;
+  d.m = fmaxf(d.m, mx);
+  if (mx > d.ref + kRefSlack) d_reref(d, mx);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) d_acc(d, bf2_to_f2(w[k]));
 }
 
 // --- drafter: 4 f32 ------------------------------------------------------------
 __device__ __forceinline__ void d_vec(DLane& d, float4 q, int v) {
   const float nc = neg_clamp();
-  const float z0 = fmaxf(q.x, nc), z1 = fmaxf(q.y, nc), z2 = fmaxf(q.z, nc), z3 = fmaxf(q.w, nc);
-  d.f2 = fmaxf(d.f2, fminf(d.f1, z0)); d.f1 = fmaxf(d.f1, z0);
-  d.f2 = fmaxf(d.f2, fminf(d.f1, z1)); d.f1 = fmaxf(d.f1, z1);
-  d.f2 = fmaxf(d.f2, fminf(d.f1, z2)); d.f1 = fmaxf(d.f1, z2);
-  d.f2 = fmaxf(d.f2, fminf(d.f1, z3)); d.f1 = fmaxf(d.f1, z3);
-  if (d.f1 > d.m) d_raise(d, d.f1, v, 4);
-  d_acc0(d, z0); d_acc1(d, z1); d_acc0(d, z2); d_acc1(d, z3);
+  const float z[4] = {fmaxf(q.x, nc), fmaxf(q.y, nc), fmaxf(q.z, nc), fmaxf(q.w, nc)};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    d.f2 = fmaxf(d.f2, fminf(d.f1, z[k]));
+    d.f1 = fmaxf(d.f1, z[k]);
+  }
+  const bool up = d.f1 > d.m;
+  d.pos = up ? v : d.pos;
+  d.posw = up ? 4 : d.posw;
+  d.m = fmaxf(d.m, d.f1);
+  if (d.f1 > d.ref + kRefSlack) d_reref(d, d.f1);
+  d_acc(d, pack2(z[0], z[1]));
+  d_acc(d, pack2(z[2], z[3]));
 }
 
-// --- target: one element --------------------------------------------------------
+// --- target -----------------------------------------------------------------------
 template <bool SAMPLED>
 __device__ __forceinline__ void t_scalar(TLane& t, float z, int v, float c, int beta) {
-  if (z > t.M) t_raise(t, z, v, 1, SAMPLED);
+  if (z > t.M) { t.pos = v; t.posw = 1; }
+  t.M = fmaxf(t.M, z);
   if (t.cnt < beta && z > c) ++t.cnt;
-  if (SAMPLED) t.s0 += ex2(fmaf(z, kLog2e, t.negML));
+  if (SAMPLED) {
+    if (z > t.ref + kRefSlack) t_reref(t, z);
+    t_acc(t, pack2(z, -pos_inf()));
+  }
 }
 
 template <bool SAMPLED>
 __device__ __forceinline__ void t_vec(TLane& t, uint4 q, int v, float c, int beta) {
-  const uint32_t a = bmax2(bmax2(q.x, q.y), bmax2(q.z, q.w));
+  const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+  const uint32_t a = bmax2(bmax2(w[0], w[1]), bmax2(w[2], w[3]));
   const float vmax = fmaxf(bf_lo(a), bf_hi(a));
-  if (vmax > t.M) t_raise(t, vmax, v, 8, SAMPLED);
-  if (t.cnt < beta && vmax > c) {
-    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+  const bool up = vmax > t.M;
+  t.pos = up ? v : t.pos;
+  t.posw = up ? 8 : t.posw;
+  t.M = fmaxf(t.M, vmax);
+  if (vmax > t.thr) {          // PAPER rule, rank gate: count logits above the draft's
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      t.cnt += (bf_lo(w[k]) > c) + (bf_hi(w[k]) > c);
-    }
+    for (int k = 0; k < 4; ++k) t.cnt += (bf_lo(w[k]) > c) + (bf_hi(w[k]) > c);
+    if (t.cnt >= beta) t.thr = pos_inf();
   }
   if (SAMPLED) {
-    const float n = t.negML;
-    t.s0 += ex2(fmaf(bf_lo(q.x), kLog2e, n)); t.s1 += ex2(fmaf(bf_hi(q.x), kLog2e, n));
-    t.s0 += ex2(fmaf(bf_lo(q.y), kLog2e, n)); t.s1 += ex2(fmaf(bf_hi(q.y), kLog2e, n));
-    t.s0 += ex2(fmaf(bf_lo(q.z), kLog2e, n)); t.s1 += ex2(fmaf(bf_hi(q.z), kLog2e, n));
-    t.s0 += ex2(fmaf(bf_lo(q.w), kLog2e, n)); t.s1 += ex2(fmaf(bf_hi(q.w), kLog2e, n));
+    if (vmax > t.ref + kRefSlack) t_reref(t, vmax);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) t_acc(t, bf2_to_f2(w[k]));
   }
 }
 
 template <bool SAMPLED>
 __device__ __forceinline__ void t_vec(TLane& t, float4 q, int v, float c, int beta) {
-  const float vmax = fmaxf(fmaxf(q.x, q.y), fmaxf(q.z, q.w));
-  if (vmax > t.M) t_raise(t, vmax, v, 4, SAMPLED);
-  if (t.cnt < beta && vmax > c) t.cnt += (q.x > c) + (q.y > c) + (q.z > c) + (q.w > c);
-  if (SAMPLED) {
-    const float n = t.negML;
-    t.s0 += ex2(fmaf(q.x, kLog2e, n)); t.s1 += ex2(fmaf(q.y, kLog2e, n));
-    t.s0 += ex2(fmaf(q.z, kLog2e, n)); t.s1 += ex2(fmaf(q.w, kLog2e, n));
+  const float z[4] = {q.x, q.y, q.z, q.w};
+  const float vmax = fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3]));
+  const bool up = vmax > t.M;
+  t.pos = up ? v : t.pos;
+  t.posw = up ? 4 : t.posw;
+  t.M = fmaxf(t.M, vmax);
+  if (vmax > t.thr) {
+    t.cnt += (z[0] > c) + (z[1] > c) + (z[2] > c) + (z[3] > c);
+    if (t.cnt >= beta) t.thr = pos_inf();
   }
+  if (SAMPLED) {
+    if (vmax > t.ref + kRefSlack) t_reref(t, vmax);
+    t_acc(t, pack2(z[0], z[1]));
+    t_acc(t, pack2(z[2], z[3]));
+  }
+}
+
+// s and t of a drafter lane relative to its exact maximum m
+__device__ __forceinline__ void d_final(const DLane& d, float& s, float& t2) {
+  const float dd = __fsub_rn(-lo32f(d.negrL), mlog2e(d.m));   // (ref - m) log2e <= 0
+  const float sc = ex2(dd);
+  const float s0 = lo32f(d.s) + hi32f(d.s);
+  s = s0 * sc;
+  t2 = sc * fmaf(s0, dd, lo32f(d.t) + hi32f(d.t));
+}
+__device__ __forceinline__ float t_final(const TLane& t) {
+  return (lo32f(t.s) + hi32f(t.s)) * ex2(__fsub_rn(-lo32f(t.negrL), mlog2e(t.M)));
 }
 
 template <typename T> struct VecT;
@@ -270,6 +309,11 @@ __device__ __forceinline__ float warp_max(float x) {
   for (int o = 16; o; o >>= 1) x = fmaxf(x, __shfl_xor_sync(kFull, x, o));
   return x;
 }
+__device__ __forceinline__ float warp_min(float x) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) x = fminf(x, __shfl_xor_sync(kFull, x, o));
+  return x;
+}
 __device__ __forceinline__ int warp_min_i(int x) {
 #pragma unroll
   for (int o = 16; o; o >>= 1) x = min(x, __shfl_xor_sync(kFull, x, o));
@@ -290,44 +334,82 @@ __device__ __forceinline__ float warp_sum_f(float x) {
 struct DRed { float m, s, t2, top2; int idx; };
 struct TRed { float m, s; int idx, cnt; };
 
+__device__ __forceinline__ DRed dred_empty() { return DRed{kNegInit, 0.f, 0.f, kNegInit, kIntMax}; }
+__device__ __forceinline__ TRed tred_empty() { return TRed{kNegInit, 0.f, kIntMax, 0}; }
+
 // Merge per-lane drafter statistics (m, s, t2 relative to m, top2, idx).
-__device__ __forceinline__ DRed reduce_d(float m, float s, float t2, float top2, int idx) {
+__device__ __forceinline__ DRed reduce_d(const DRed& x) {
   DRed r;
-  r.m = warp_max(m);
-  const float ML = r.m * kLog2e;
-  const float dd = m * kLog2e - ML;
+  r.m = warp_max(x.m);
+  const float ML = mlog2e(r.m);
+  const float dd = __fsub_rn(mlog2e(x.m), ML);
   const float sc = ex2(dd);
-  const float s_ = s * sc;
-  const float t_ = sc * fmaf(s, dd, t2);
-  r.s = warp_sum_f(s_);
-  r.t2 = warp_sum_f(t_);
-  r.idx = warp_min_i(m == r.m ? idx : 0x7FFFFFFF);
-  r.top2 = warp_max((m == r.m && idx == r.idx) ? top2 : m);
+  r.s = warp_sum_f(x.s * sc);
+  r.t2 = warp_sum_f(sc * fmaf(x.s, dd, x.t2));
+  r.idx = warp_min_i(x.m == r.m ? x.idx : kIntMax);
+  r.top2 = warp_max((x.m == r.m && x.idx == r.idx) ? x.top2 : x.m);
   return r;
 }
-__device__ __forceinline__ TRed reduce_t(float m, float s, int idx, int cnt) {
+__device__ __forceinline__ TRed reduce_t(const TRed& x) {
   TRed r;
-  r.m = warp_max(m);
-  const float sc = ex2(m * kLog2e - r.m * kLog2e);
-  r.s = warp_sum_f(s * sc);
-  r.idx = warp_min_i(m == r.m ? idx : 0x7FFFFFFF);
-  r.cnt = warp_sum_i(cnt);
+  r.m = warp_max(x.m);
+  const float sc = ex2(__fsub_rn(mlog2e(x.m), mlog2e(r.m)));
+  r.s = warp_sum_f(x.s * sc);
+  r.idx = warp_min_i(x.m == r.m ? x.idx : kIntMax);
+  r.cnt = warp_sum_i(x.cnt);
   return r;
+}
+
+// Lane-local merge of two partial statistics (used when a row has more
+// partials than a warp has lanes).
+__device__ __forceinline__ void fold_d(DRed& a, const DRed& b) {
+  const float M = fmaxf(a.m, b.m);
+  const float ML = mlog2e(M);
+  const float da = __fsub_rn(mlog2e(a.m), ML), db = __fsub_rn(mlog2e(b.m), ML);
+  const float sa = ex2(da), sb = ex2(db);
+  const float t2 = sa * fmaf(a.s, da, a.t2) + sb * fmaf(b.s, db, b.t2);
+  const float s = a.s * sa + b.s * sb;
+  if (a.m > b.m) {
+    a.top2 = fmaxf(a.top2, b.m);
+  } else if (b.m > a.m) {
+    a.top2 = fmaxf(b.top2, a.m);
+    a.idx = b.idx;
+  } else {
+    a.top2 = a.m;
+    a.idx = min(a.idx, b.idx);
+  }
+  a.m = M;
+  a.s = s;
+  a.t2 = t2;
+}
+__device__ __forceinline__ void fold_t(TRed& a, const TRed& b) {
+  const float M = fmaxf(a.m, b.m);
+  const float ML = mlog2e(M);
+  const float s = a.s * ex2(__fsub_rn(mlog2e(a.m), ML)) + b.s * ex2(__fsub_rn(mlog2e(b.m), ML));
+  if (b.m > a.m) a.idx = b.idx;
+  else if (b.m == a.m) a.idx = min(a.idx, b.idx);
+  a.m = M;
+  a.s = s;
+  a.cnt += b.cnt;
 }
 
 // ---------------------------------------------------------------------------
 // work split
 // ---------------------------------------------------------------------------
 
-__device__ __forceinline__ int64_t min_len(int V) {
-  const int64_t a = (int64_t)V / 24 + 64;
-  return a > 1024 ? a : 1024;
-}
-__device__ __forceinline__ int eff_warps(int64_t N, int V, int nwarps) {
-  int64_t w = N / min_len(V);
+__device__ __forceinline__ int eff_warps(int64_t N, int64_t min_len, int nwarps) {
+  int64_t w = N / min_len;
   if (w < 1) w = 1;
   if (w > nwarps) w = nwarps;
   return (int)w;
+}
+__device__ __forceinline__ int64_t stream_min_len(int V) {
+  const int64_t a = (int64_t)V / 64 + 64;
+  return a > 2048 ? a : 2048;
+}
+__device__ __forceinline__ int64_t stream_cta_min_len(int V) {
+  const int64_t a = (int64_t)V / 16 + 64;
+  return a > 16384 ? a : 16384;
 }
 __device__ __forceinline__ int64_t split_start(int w, int64_t N, int W, int vec) {
   if (w >= W) return N;
@@ -363,7 +445,6 @@ __device__ __forceinline__ void map_row(const StreamArgs& a, const int* pref, in
   i = ar - pref[lo];
 }
 
-template <typename T>
 __device__ __forceinline__ int checked_token(const StreamArgs& a, int r) {
   int tok = __ldg(a.tokens + r);
   if (tok < 0 || tok >= a.V) {
@@ -371,6 +452,32 @@ __device__ __forceinline__ int checked_token(const StreamArgs& a, int r) {
     tok = 0;
   }
   return tok;
+}
+
+// Geometry of one segment: row elements [v0, v1), with the 16-byte aligned
+// body [va, vb) (a whole number of vectors) between a head and a tail.
+struct Seg {
+  int ar, b, i, r;
+  int v0, v1, va, vb;
+};
+
+template <typename T>
+__device__ __forceinline__ Seg make_seg(const StreamArgs& a, const int* pref, int64_t e, int64_t e_end,
+                                        const void* base) {
+  constexpr int VEC = Elem<T>::kVec;
+  Seg s;
+  s.ar = (int)(e / a.V);
+  s.v0 = (int)(e - (int64_t)s.ar * a.V);
+  const int len = (int)min((int64_t)(a.V - s.v0), e_end - e);
+  s.v1 = s.v0 + len;
+  map_row(a, pref, s.ar, s.b, s.i);
+  s.r = s.b * a.K + s.i;
+  const uintptr_t addr = (uintptr_t)((const T*)base + (size_t)s.r * (size_t)a.V + s.v0);
+  const int mis = (int)((addr & 15) / sizeof(T));
+  const int head = mis ? min(VEC - mis, len) : 0;
+  s.va = s.v0 + head;
+  s.vb = s.va + ((s.v1 - s.va) / VEC) * VEC;
+  return s;
 }
 
 // ---------------------------------------------------------------------------
@@ -446,10 +553,10 @@ __device__ void row_results(const StreamArgs& a, int r, int b, int i, const DRed
   const Workspace& W = a.ws;
   float C = 0.f, MLd = 0.f, Sd = 1.f;
   if (MODE != kModeVerify) {
-    MLd = d.m * kLog2e;
+    MLd = mlog2e(d.m);
     Sd = d.s;
     const float H = kLn2 * (log2f(d.s) - d.t2 / d.s);
-    const float margin = (d.top2 <= neg_clamp()) ? __int_as_float(0x7F800000) : d.m - d.top2;
+    const float margin = (d.top2 <= neg_clamp()) ? pos_inf() : d.m - d.top2;
     const float psm = (1.0f - exp2f(fmaf(d.top2, kLog2e, -MLd))) / d.s;
     const float Vf = (float)a.V;
     const float c_ent = 1.0f - H / logf(Vf);
@@ -471,12 +578,12 @@ __device__ void row_results(const StreamArgs& a, int r, int b, int i, const DRed
                                         : a.tau_base + a.gamma * C;
     const bool rank_ok = a.beta_rank <= 0 || t.cnt < a.beta_rank;
     bool acc;
-    const float MLt = t.m * kLog2e;
+    const float MLt = mlog2e(t.m);
     if (!SAMPLED) {
       const float gap = t.m - c_tgt;
       acc = rank_ok && gap <= tau;
     } else {
-      const int tok = checked_token<T>(a, r);
+      const int tok = checked_token(a, r);
       const float zd = Elem<T>::load((const T*)a.draft + (size_t)r * a.V + tok);
       const float p = exp2f(fmaf(c_tgt, kLog2e, -MLt)) / t.s;
       float q;
@@ -503,28 +610,242 @@ __device__ void row_results(const StreamArgs& a, int r, int b, int i, const DRed
 // ---------------------------------------------------------------------------
 // the streaming kernel
 // ---------------------------------------------------------------------------
+//
+// Every warp owns one contiguous slice of the stream.  Within each segment
+// (the part of one row inside the slice) a lane's 16-byte vectors are those
+// with index lane + 32 t; they are staged kStagesRing stages ahead, CMSD_UNROLL
+// vectors of each tensor per stage, by asynchronous global->shared copies
+// into the lane's own slots, and read back by the same lane, so no lane waits
+// on another and the waits (cp.async.wait_group) block in hardware.  A
+// segment's unaligned head and tail (under 16 bytes each) are read directly.
+// At the end of a segment the warp reduces its lanes and writes one Partial;
+// the warp that completes a row merges the row and, when it completes a
+// sequence, runs the sequence epilogue.  Warps never wait on each other.
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+#ifndef CMSD_MIN_BLOCKS
+#define CMSD_MIN_BLOCKS 3
+#endif
+
+// Running state of the segment a warp is reducing.
+template <typename T>
+struct SegState {
+  DLane d;
+  TLane t;
+  float c;          // target logit at the drafted token
+};
 
 template <typename T, int MODE, bool SAMPLED>
-__global__ void __launch_bounds__(kThreads) stream_kernel(const StreamArgs a) {
+__device__ __forceinline__ void seg_begin(SegState<T>& ss, float c_tgt, int beta) {
+  dlane_init(ss.d);
+  tlane_init(ss.t, c_tgt, beta);
+  ss.c = c_tgt;
+}
+
+// End of a segment (row ar / storage row r / sequence b, position i, len
+// logits): warp-reduce, publish the partial, and merge the row / run the
+// sequence epilogue if this warp completes them.
+template <typename T, int MODE, bool SAMPLED>
+__device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, int b, int i, int len,
+                           int64_t N, int Weff, int w, int lane) {
+  const T* dp = (const T*)a.draft + (size_t)r * (size_t)a.V;
+  const T* tp = (MODE != kModeConf) ? (const T*)a.target + (size_t)r * (size_t)a.V : nullptr;
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   constexpr int VEC = Elem<T>::kVec;
-  using V4 = typename VecT<T>::type;
-  extern __shared__ int s_pref[];
+  const Workspace& W = a.ws;
+  DRed dr = dred_empty();
+  TRed tr = tred_empty();
+  if (HAS_D) {
+    const DLane& d = ss.d;
+    float top1 = d.f1, top2 = d.f2;
+    if (sizeof(T) == 2) {
+      const float a1 = bf_lo(d.T1), a2 = bf_lo(d.T2), b1 = bf_hi(d.T1), b2 = bf_hi(d.T2);
+      const float u1 = fmaxf(a1, b1), u2 = fmaxf(fminf(a1, b1), fmaxf(a2, b2));
+      top2 = fmaxf(fminf(u1, top1), fmaxf(u2, top2));
+      top1 = fmaxf(u1, top1);
+    }
+    float s, t2;
+    d_final(d, s, t2);
+    // only lanes holding the segment maximum resolve their exact index
+    const float M = warp_max(d.m);
+    const int idx = (d.m == M && d.posw) ? first_equal<T>(dp, d.pos, d.posw, d.m, true) : kIntMax;
+    dr = reduce_d(DRed{d.m, s, t2, top2, idx});
+  }
+  if (HAS_T) {
+    const TLane& t = ss.t;
+    const float M = warp_max(t.M);
+    const int idx = (t.M == M && t.posw) ? first_equal<T>(tp, t.pos, t.posw, t.M, false) : kIntMax;
+    tr = reduce_t(TRed{t.M, SAMPLED ? t_final(t) : 0.f, idx, t.cnt});
+  }
+  if (lane == 0) {
+    Partial p;
+    p.d_m = dr.m; p.d_s = dr.s; p.d_t2 = dr.t2; p.d_top2 = dr.top2; p.d_idx = dr.idx;
+    p.t_m = tr.m; p.t_s = tr.s; p.t_idx = tr.idx; p.t_cnt = tr.cnt;
+    p.pad[0] = p.pad[1] = p.pad[2] = 0;
+    W.part[ar + w] = p;
+  }
+  __threadfence();
+  int old = 0;
+  if (lane == 0) old = atomicAdd(W.row_done + r, len);
+  old = __shfl_sync(kFull, old, 0);
+  if (old + len != a.V) return;
+  // -- this warp completed row r: merge every slice's partial -----------------
+  __threadfence();
+  const int wf = find_warp((int64_t)ar * a.V, N, Weff, VEC);
+  const int wl = find_warp((int64_t)ar * a.V + a.V - 1, N, Weff, VEC);
+  DRed dm = dred_empty();
+  TRed tm = tred_empty();
+  for (int k = wf + lane; k <= wl; k += 32) {
+    const float4* src = reinterpret_cast<const float4*>(W.part + ar + k);
+    const float4 x0 = __ldcg(src), x1 = __ldcg(src + 1), x2 = __ldcg(src + 2);
+    if (HAS_D) fold_d(dm, DRed{x0.x, x0.y, x0.z, x0.w, __float_as_int(x1.x)});
+    if (HAS_T) fold_t(tm, TRed{x1.y, x1.z, __float_as_int(x1.w), __float_as_int(x2.x)});
+  }
+  if (HAS_D) dr = reduce_d(dm);
+  if (HAS_T) tr = reduce_t(tm);
+  if (lane == 0) {
+    W.row_done[r] = 0;
+    row_results<T, MODE, SAMPLED>(a, r, b, i, dr, tr, ss.c);
+  }
+  __threadfence();
+  const int kb = k_of(a, b);
+  int sold = 0;
+  if (lane == 0) sold = atomicAdd(W.seq_done + b, 1);
+  sold = __shfl_sync(kFull, sold, 0);
+  if (sold + 1 == kb) {
+    __threadfence();
+    seq_epilogue<MODE, SAMPLED>(a, b, kb, lane);
+  }
+}
+
+template <typename T>
+__device__ __forceinline__ float target_at_token(const StreamArgs& a, int r) {
+  return Elem<T>::load((const T*)a.target + (size_t)r * (size_t)a.V + checked_token(a, r));
+}
+
+// ---- one segment body, pipelined ----------------------------------------------
+// The lane's vectors of the aligned body [va, vb) are j = lane + 32 t,
+// t = 0, 1, ...; stage s holds t in [s*U, s*U + U).  Stages are copied
+// kStagesRing ahead with asynchronous copies into the lane's own slots and
+// read back by the same lane.
+#ifndef CMSD_UNROLL
+#define CMSD_UNROLL 2
+#endif
+template <typename T, int MODE, bool SAMPLED>
+__device__ __forceinline__ void walk_body(SegState<T>& ss, const T* dp, const T* tp, int va, int vb, int beta,
+                                          unsigned char* lane_ring, int lane) {
+  constexpr bool HAS_D = MODE != kModeVerify;
+  constexpr bool HAS_T = MODE != kModeConf;
+  constexpr int VEC = Elem<T>::kVec;
+  constexpr int U = CMSD_UNROLL;
+  constexpr int SLOT = U * 2 * 512;                  // bytes of one stage of one warp
+  const int nvec = (vb - va) / VEC;
+  if (nvec <= 0) return;
+  const int nt = nvec > lane ? (nvec - lane + 31) / 32 : 0;   // this lane's vectors
+  const int nst = (nt + U - 1) / U;                            // this lane's stages
+  const unsigned char* gd = reinterpret_cast<const unsigned char*>(dp + va) + 16 * lane;
+  const unsigned char* gt = HAS_T ? reinterpret_cast<const unsigned char*>(tp + va) + 16 * lane : nullptr;
+  const uint32_t ring_s = smem_u32(lane_ring);
+  // issue stage s (vectors t = s*U + u of this lane) into slot s % kStagesRing
+  auto issue = [&](int s, uint32_t slot_s) {
+    if (s < nst) {
+      const int t0 = s * U;
+      const size_t go = (size_t)t0 * 512;
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (t0 + u < nt) {
+          if (HAS_D) cp_async16(slot_s + 512u * u, gd + go + 512 * u);
+          if (HAS_T) cp_async16(slot_s + 512u * (U + u), gt + go + 512 * u);
+        }
+      }
+    }
+    cp_async_commit();
+  };
+#pragma unroll
+  for (int s = 0; s < kStagesRing; ++s) issue(s, ring_s + (uint32_t)(s * SLOT));
+  int slot = 0;
+  for (int s = 0; s < nst; ++s) {
+    cp_async_wait<kStagesRing - 1>();
+    const unsigned char* sl = lane_ring + slot * SLOT;
+    const int t0 = s * U;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (t0 + u < nt) {
+        const int v = va + (lane + 32 * (t0 + u)) * VEC;
+        if (HAS_D) d_vec(ss.d, as_vec<T>(*reinterpret_cast<const uint4*>(sl + 512 * u)), v);
+        if (HAS_T) t_vec<SAMPLED>(ss.t, as_vec<T>(*reinterpret_cast<const uint4*>(sl + 512 * (U + u))), v, ss.c, beta);
+      }
+    }
+    issue(s + kStagesRing, ring_s + (uint32_t)(slot * SLOT));
+    slot = slot + 1 == kStagesRing ? 0 : slot + 1;
+  }
+  cp_async_wait<0>();
+}
+
+// ---- a warp's slice, segment by segment ------------------------------------------
+template <typename T, int MODE, bool SAMPLED>
+__device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_begin, int64_t e_end,
+                           int64_t N, int Weff, int w, int lane, unsigned char* lane_ring) {
+  constexpr bool HAS_D = MODE != kModeVerify;
+  constexpr bool HAS_T = MODE != kModeConf;
+  const int beta = a.beta_rank > 0 ? a.beta_rank : 0;
+  const void* base = HAS_D ? a.draft : a.target;
+  float c_next = 0.f;
+  if (HAS_T) c_next = target_at_token<T>(a, make_seg<T>(a, s_pref, e_begin, e_end, base).r);
+  for (int64_t e0 = e_begin; e0 < e_end;) {
+    const Seg sg = make_seg<T>(a, s_pref, e0, e_end, base);
+    const int len = sg.v1 - sg.v0;
+    e0 += len;
+    const size_t rowoff = (size_t)sg.r * (size_t)a.V;
+    const T* dp = (const T*)a.draft + rowoff;
+    const T* tp = HAS_T ? (const T*)a.target + rowoff : nullptr;
+    SegState<T> ss;
+    seg_begin<T, MODE, SAMPLED>(ss, c_next, beta);
+    if (HAS_T && e0 < e_end) c_next = target_at_token<T>(a, make_seg<T>(a, s_pref, e0, e_end, base).r);
+    if (lane < sg.va - sg.v0) {
+      const int v = sg.v0 + lane;
+      if (HAS_D) d_scalar(ss.d, Elem<T>::load(dp + v), v);
+      if (HAS_T) t_scalar<SAMPLED>(ss.t, Elem<T>::load(tp + v), v, ss.c, beta);
+    }
+    walk_body<T, MODE, SAMPLED>(ss, dp, tp, sg.va, sg.vb, beta, lane_ring, lane);
+    if (lane < sg.v1 - sg.vb) {
+      const int v = sg.vb + lane;
+      if (HAS_D) d_scalar(ss.d, Elem<T>::load(dp + v), v);
+      if (HAS_T) t_scalar<SAMPLED>(ss.t, Elem<T>::load(tp + v), v, ss.c, beta);
+    }
+    seg_finish<T, MODE, SAMPLED>(a, ss, sg.ar, sg.r, sg.b, sg.i, len, N, Weff, w, lane);
+  }
+}
+
+template <typename T, int MODE, bool SAMPLED>
+__global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const StreamArgs a) {
+  constexpr bool HAS_D = MODE != kModeVerify;
+  constexpr bool HAS_T = MODE != kModeConf;
+  constexpr int VEC = Elem<T>::kVec;
+  extern __shared__ __align__(128) unsigned char smem[];
 
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const Workspace& W = a.ws;
+  const bool ragged = a.k_row != nullptr;
+  int* s_pref = reinterpret_cast<int*>(smem);
+  unsigned char* my_ring = smem + stream_pref_bytes(a.B, ragged) + (size_t)warp * kStagesRing * kStageWarpBytes +
+                          16 * lane;
 
   // -- present rows: exclusive prefix of k_row (ragged windows) -------------
   int nrows;
-  if (a.k_row) {
-    // per-thread serial chunks, then a scan over thread totals
+  if (ragged) {
     const int per = (a.B + kThreads - 1) / kThreads;
     const int b0 = threadIdx.x * per;
     int tot = 0;
     for (int b = b0; b < b0 + per && b < a.B; ++b) tot += k_of(a, b);
-    // block exclusive scan of tot (warp scan + warp totals)
     int incl = tot;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -549,7 +870,7 @@ __global__ void __launch_bounds__(kThreads) stream_kernel(const StreamArgs a) {
   }
 
   // -- sequences with no present position, and k_row range errors -----------
-  if (a.k_row) {
+  if (ragged) {
     const int gt = blockIdx.x * kThreads + threadIdx.x;
     const int gn = gridDim.x * kThreads;
     for (int b = gt; b < a.B; b += gn) {
@@ -570,144 +891,12 @@ __global__ void __launch_bounds__(kThreads) stream_kernel(const StreamArgs a) {
 
   const int64_t N = (int64_t)nrows * a.V;
   if (N == 0) return;
-  const int Weff = eff_warps(N, a.V, a.nwarps);
+  const int Weff = eff_warps(N, stream_min_len(a.V), a.nwarps);
   const int w = blockIdx.x * kWarpsPerBlock + warp;
   if (w >= Weff) return;
-
-  int64_t e0 = split_start(w, N, Weff, VEC);
-  const int64_t e1 = split_start(w + 1, N, Weff, VEC);
-  const int beta = a.beta_rank > 0 ? a.beta_rank : 0;
-
-  while (e0 < e1) {
-    const int ar = (int)(e0 / a.V);
-    const int v0 = (int)(e0 - (int64_t)ar * a.V);
-    const int len = (int)min((int64_t)(a.V - v0), e1 - e0);
-    const int v1 = v0 + len;
-    int b, i;
-    map_row(a, s_pref, ar, b, i);
-    const int r = b * a.K + i;
-    const size_t rowoff = (size_t)r * (size_t)a.V;
-    const T* dp = (const T*)a.draft + rowoff;
-    const T* tp = HAS_T ? (const T*)a.target + rowoff : nullptr;
-
-    float c_tgt = 0.f;
-    if (HAS_T) c_tgt = Elem<T>::load(tp + checked_token<T>(a, r));
-
-    DLane d;
-    TLane t;
-    dlane_init(d);
-    tlane_init(t);
-
-    const T* ap = HAS_D ? dp : tp;
-    const int mis = (int)(((uintptr_t)(ap + v0) & 15) / sizeof(T));
-    const int head = mis ? min(VEC - mis, len) : 0;
-    const int va = v0 + head;
-    const int nvec = (v1 - va) / VEC;
-    const int vb = va + nvec * VEC;
-
-    if (lane < head) {
-      const int v = v0 + lane;
-      if (HAS_D) d_scalar(d, Elem<T>::load(dp + v), v);
-      if (HAS_T) t_scalar<SAMPLED>(t, Elem<T>::load(tp + v), v, c_tgt, beta);
-    }
-    {
-      const uint4* dv = reinterpret_cast<const uint4*>(dp + va);
-      const uint4* tv = HAS_T ? reinterpret_cast<const uint4*>(tp + va) : nullptr;
-      int j = lane;
-      constexpr int U = 4;
-      for (; j + (U - 1) * 32 < nvec; j += U * 32) {
-        uint4 qd[U], qt[U];
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-          if (HAS_D) qd[u] = ld_stream(dv + j + u * 32);
-          if (HAS_T) qt[u] = ld_stream(tv + j + u * 32);
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-          const int v = va + (j + u * 32) * VEC;
-          if (HAS_D) d_vec(d, as_vec<T>(qd[u]), v);
-          if (HAS_T) t_vec<SAMPLED>(t, as_vec<T>(qt[u]), v, c_tgt, beta);
-        }
-      }
-      for (; j < nvec; j += 32) {
-        const int v = va + j * VEC;
-        if (HAS_D) d_vec(d, as_vec<T>(ld_stream(dv + j)), v);
-        if (HAS_T) t_vec<SAMPLED>(t, as_vec<T>(ld_stream(tv + j)), v, c_tgt, beta);
-      }
-    }
-    if (lane < v1 - vb) {
-      const int v = vb + lane;
-      if (HAS_D) d_scalar(d, Elem<T>::load(dp + v), v);
-      if (HAS_T) t_scalar<SAMPLED>(t, Elem<T>::load(tp + v), v, c_tgt, beta);
-    }
-
-    // -- segment reduction ------------------------------------------------
-    DRed dr{};
-    TRed tr{};
-    if (HAS_D) {
-      float top1 = d.f1, top2 = d.f2;
-      if (sizeof(T) == 2) {
-        const float a1 = bf_lo(d.T1), a2 = bf_lo(d.T2), b1 = bf_hi(d.T1), b2 = bf_hi(d.T2);
-        const float u1 = fmaxf(a1, b1), u2 = fmaxf(fminf(a1, b1), fmaxf(a2, b2));
-        top2 = fmaxf(fminf(u1, top1), fmaxf(u2, top2));
-        top1 = fmaxf(u1, top1);
-      }
-      const int idx = d.posw ? first_equal<T>(dp, d.pos, d.posw, d.m, true) : 0x7FFFFFFF;
-      dr = reduce_d(d.m, d.s0 + d.s1, d.t0 + d.t1, top2, idx);
-    }
-    if (HAS_T) {
-      const int idx = t.posw ? first_equal<T>(tp, t.pos, t.posw, t.M, false) : 0x7FFFFFFF;
-      tr = reduce_t(t.M, t.s0 + t.s1, idx, t.cnt);
-    }
-
-    Partial* slot = W.part + ar + w;
-    if (lane == 0) {
-      Partial p;
-      p.d_m = dr.m; p.d_s = dr.s; p.d_t2 = dr.t2; p.d_top2 = dr.top2; p.d_idx = dr.idx;
-      p.t_m = tr.m; p.t_s = tr.s; p.t_idx = tr.idx; p.t_cnt = tr.cnt;
-      p.pad[0] = p.pad[1] = p.pad[2] = 0;
-      *slot = p;
-    }
-    __threadfence();
-    int old = 0;
-    if (lane == 0) old = atomicAdd(W.row_done + r, len);
-    old = __shfl_sync(kFull, old, 0);
-
-    if (old + len == a.V) {
-      // -- this warp completed row r: merge every segment's partial ----------
-      __threadfence();
-      const int wf = find_warp((int64_t)ar * a.V, N, Weff, VEC);
-      const int wl = find_warp((int64_t)ar * a.V + a.V - 1, N, Weff, VEC);
-      const int np = wl - wf + 1;      // <= 26 by the minimum slice length
-      Partial p;
-      if (lane < np) {
-        const float4* src = reinterpret_cast<const float4*>(W.part + ar + wf + lane);
-        const float4 x0 = __ldcg(src), x1 = __ldcg(src + 1), x2 = __ldcg(src + 2);
-        p.d_m = x0.x; p.d_s = x0.y; p.d_t2 = x0.z; p.d_top2 = x0.w;
-        p.d_idx = __float_as_int(x1.x); p.t_m = x1.y; p.t_s = x1.z; p.t_idx = __float_as_int(x1.w);
-        p.t_cnt = __float_as_int(x2.x);
-      } else {
-        p.d_m = kNegInit; p.d_s = 0.f; p.d_t2 = 0.f; p.d_top2 = kNegInit; p.d_idx = 0x7FFFFFFF;
-        p.t_m = kNegInit; p.t_s = 0.f; p.t_idx = 0x7FFFFFFF; p.t_cnt = 0;
-      }
-      if (HAS_D) dr = reduce_d(p.d_m, p.d_s, p.d_t2, p.d_top2, p.d_idx);
-      if (HAS_T) tr = reduce_t(p.t_m, p.t_s, p.t_idx, p.t_cnt);
-      if (lane == 0) {
-        W.row_done[r] = 0;
-        row_results<T, MODE, SAMPLED>(a, r, b, i, dr, tr, c_tgt);
-      }
-      __threadfence();
-      const int kb = k_of(a, b);
-      int sold = 0;
-      if (lane == 0) sold = atomicAdd(W.seq_done + b, 1);
-      sold = __shfl_sync(kFull, sold, 0);
-      if (sold + 1 == kb) {
-        __threadfence();
-        seq_epilogue<MODE, SAMPLED>(a, b, kb, lane);
-      }
-    }
-    e0 += len;
-  }
+  const int64_t e_begin = split_start(w, N, Weff, VEC);
+  const int64_t e_end = split_start(w + 1, N, Weff, VEC);
+  walk_slice<T, MODE, SAMPLED>(a, s_pref, e_begin, e_end, N, Weff, w, lane, my_ring);
 }
 
 // ---------------------------------------------------------------------------
@@ -721,30 +910,63 @@ struct Race {
   U4 words;
 };
 
-__device__ __forceinline__ void race_elem(Race& rc, float zt, float zd, int v, float MLt, float invSt,
-                                          float MLd, float invSd, uint32_t b, uint32_t n,
-                                          uint32_t cw, uint32_t k0, uint32_t k1) {
-  const float p = ex2(fmaf(zt, kLog2e, -MLt)) * invSt;
-  const float q = ex2(fmaf(zd, kLog2e, -MLd)) * invSd;
+__device__ __forceinline__ uint32_t pick(const U4& w, uint32_t sel) {
+  return sel == 0 ? w.x : sel == 1 ? w.y : sel == 2 ? w.z : w.w;
+}
+
+// One candidate of the race: r = p - q; if r > 0 its key is E / r with
+// E = -log(1 - u).  E >= u, so entries with u >= key * r cannot beat the
+// current best and skip the logarithm.
+__device__ __forceinline__ void race_try(Race& rc, float p, float q, uint32_t word, int v) {
   const float rr = p - q;
   if (rr > 0.f) {
-    const uint32_t g = (uint32_t)v >> 2;
-    if (g != rc.grp) {
-      rc.words = philox4x32_10(U4{g, b, n, cw}, k0, k1);
-      rc.grp = g;
-    }
-    const uint32_t sel = (uint32_t)v & 3u;
-    const uint32_t word = sel == 0 ? rc.words.x : sel == 1 ? rc.words.y : sel == 2 ? rc.words.z : rc.words.w;
     const float u = word_to_unit(word);
-    // E = -log(1 - u) >= u: skip entries that cannot beat the current best
     if (u < rc.key * rr) {
-      const float E = -log1pf(-u);
-      const float key = E / rr;
+      const float key = -log1pf(-u) / rr;
       if (key < rc.key) {
         rc.key = key;
         rc.idx = v;
       }
     }
+  }
+}
+
+// Element-at-a-time form (row heads/tails, and rows whose vectors do not start
+// on a multiple of 4): the Philox block of group v >> 2 is cached per lane.
+__device__ __forceinline__ void race_elem(Race& rc, float zt, float zd, int v, float MLt, float invSt,
+                                          float MLd, float invSd, uint32_t b, uint32_t n,
+                                          uint32_t cw, uint32_t k0, uint32_t k1) {
+  const float p = ex2(fmaf(zt, kLog2e, -MLt)) * invSt;
+  const float q = ex2(fmaf(zd, kLog2e, -MLd)) * invSd;
+  if (p > q) {
+    const uint32_t g = (uint32_t)v >> 2;
+    if (g != rc.grp) {
+      rc.words = philox4x32_10(U4{g, b, n, cw}, k0, k1);
+      rc.grp = g;
+    }
+    race_try(rc, p, q, pick(rc.words, (uint32_t)v & 3u), v);
+  }
+}
+
+// Four consecutive entries v .. v+3 (v a multiple of 4): one Philox block,
+// generated only when some entry of the group has p > q.
+__device__ __forceinline__ void race_group(Race& rc, const float (&zt)[4], const float (&zd)[4], int v,
+                                           float MLt, float invSt, float MLd, float invSd, uint32_t b,
+                                           uint32_t n, uint32_t cw, uint32_t k0, uint32_t k1) {
+  float p[4], q[4];
+  bool any = false;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    p[k] = ex2(fmaf(zt[k], kLog2e, -MLt)) * invSt;
+    q[k] = ex2(fmaf(zd[k], kLog2e, -MLd)) * invSd;
+    any |= p[k] > q[k];
+  }
+  if (any) {
+    const U4 rw = philox4x32_10(U4{(uint32_t)v >> 2, b, n, cw}, k0, k1);
+    race_try(rc, p[0], q[0], rw.x, v);
+    race_try(rc, p[1], q[1], rw.y, v + 1);
+    race_try(rc, p[2], q[2], rw.z, v + 2);
+    race_try(rc, p[3], q[3], rw.w, v + 3);
   }
 }
 
@@ -758,7 +980,7 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) 
   R = R < 0 ? 0 : (R > a.B ? a.B : R);
   const int64_t N = (int64_t)R * a.V;
   if (N > 0) {
-    const int Weff = eff_warps(N, a.V, a.nwarps);
+    const int Weff = eff_warps(N, 1024, a.nwarps);
     const int w = blockIdx.x * kWarpsPerBlock + warp;
     if (w < Weff) {
       int64_t e0 = split_start(w, N, Weff, VEC);
@@ -781,8 +1003,8 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) 
         const T* tp = (const T*)a.target + rowoff;
 
         Race rc;
-        rc.key = __int_as_float(0x7F800000);
-        rc.idx = 0x7FFFFFFF;
+        rc.key = pos_inf();
+        rc.idx = kIntMax;
         rc.grp = 0xFFFFFFFFu;
         rc.words = U4{0, 0, 0, 0};
 
@@ -798,24 +1020,43 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) 
         }
         const uint4* dv = reinterpret_cast<const uint4*>(dp + va);
         const uint4* tv = reinterpret_cast<const uint4*>(tp + va);
-        for (int j = lane; j < nvec; j += 32) {
-          const uint4 qd = ld_stream(dv + j), qt = ld_stream(tv + j);
-          const int v = va + j * VEC;
-          if (sizeof(T) == 2) {
-            const uint32_t wd[4] = {qd.x, qd.y, qd.z, qd.w};
-            const uint32_t wt[4] = {qt.x, qt.y, qt.z, qt.w};
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              race_elem(rc, bf_lo(wt[k]), bf_lo(wd[k]), v + 2 * k, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
-              race_elem(rc, bf_hi(wt[k]), bf_hi(wd[k]), v + 2 * k + 1, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
+        if ((va & 3) == 0) {
+          for (int j = lane; j < nvec; j += 32) {
+            const uint4 qd = ld_stream(dv + j), qt = ld_stream(tv + j);
+            const int v = va + j * VEC;
+            if (sizeof(T) == 2) {
+              const float zt0[4] = {bf_lo(qt.x), bf_hi(qt.x), bf_lo(qt.y), bf_hi(qt.y)};
+              const float zd0[4] = {bf_lo(qd.x), bf_hi(qd.x), bf_lo(qd.y), bf_hi(qd.y)};
+              race_group(rc, zt0, zd0, v, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
+              const float zt1[4] = {bf_lo(qt.z), bf_hi(qt.z), bf_lo(qt.w), bf_hi(qt.w)};
+              const float zd1[4] = {bf_lo(qd.z), bf_hi(qd.z), bf_lo(qd.w), bf_hi(qd.w)};
+              race_group(rc, zt1, zd1, v + 4, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
+            } else {
+              const float zt[4] = {__uint_as_float(qt.x), __uint_as_float(qt.y), __uint_as_float(qt.z),
+                                   __uint_as_float(qt.w)};
+              const float zd[4] = {__uint_as_float(qd.x), __uint_as_float(qd.y), __uint_as_float(qd.z),
+                                   __uint_as_float(qd.w)};
+              race_group(rc, zt, zd, v, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
             }
-          } else {
+          }
+        } else {
+          for (int j = lane; j < nvec; j += 32) {
+            const uint4 qd = ld_stream(dv + j), qt = ld_stream(tv + j);
+            const int v = va + j * VEC;
             const uint32_t wd[4] = {qd.x, qd.y, qd.z, qd.w};
             const uint32_t wt[4] = {qt.x, qt.y, qt.z, qt.w};
+            if (sizeof(T) == 2) {
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-              race_elem(rc, __uint_as_float(wt[k]), __uint_as_float(wd[k]), v + k, ts.x, invSt, ds.x,
-                        invSd, b, n, cw, k0, k1);
+              for (int k = 0; k < 4; ++k) {
+                race_elem(rc, bf_lo(wt[k]), bf_lo(wd[k]), v + 2 * k, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
+                race_elem(rc, bf_hi(wt[k]), bf_hi(wd[k]), v + 2 * k + 1, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
+              }
+            } else {
+#pragma unroll
+              for (int k = 0; k < 4; ++k)
+                race_elem(rc, __uint_as_float(wt[k]), __uint_as_float(wd[k]), v + k, ts.x, invSt, ds.x,
+                          invSd, b, n, cw, k0, k1);
+            }
           }
         }
         if (lane < v1 - vb) {
@@ -824,10 +1065,8 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) 
                     b, n, cw, k0, k1);
         }
         // warp: smallest key, lowest index among equal keys
-        float kmin = rc.key;
-#pragma unroll
-        for (int o = 16; o; o >>= 1) kmin = fminf(kmin, __shfl_xor_sync(kFull, kmin, o));
-        const int imin = warp_min_i(rc.key == kmin ? rc.idx : 0x7FFFFFFF);
+        const float kmin = warp_min(rc.key);
+        const int imin = warp_min_i(rc.key == kmin ? rc.idx : kIntMax);
         if (lane == 0) W.rpart[rr_ + w] = RacePartial{kmin, imin};
         __threadfence();
         int old = 0;
@@ -837,20 +1076,21 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) 
           __threadfence();
           const int wf = find_warp((int64_t)rr_ * a.V, N, Weff, VEC);
           const int wl = find_warp((int64_t)rr_ * a.V + a.V - 1, N, Weff, VEC);
-          float key = __int_as_float(0x7F800000);
-          int idx = 0x7FFFFFFF;
-          if (lane < wl - wf + 1) {
-            const float2 x = __ldcg(reinterpret_cast<const float2*>(W.rpart + rr_ + wf + lane));
-            key = x.x;
-            idx = __float_as_int(x.y);
+          float key = pos_inf();
+          int idx = kIntMax;
+          for (int k = wf + lane; k <= wl; k += 32) {
+            const float2 x = __ldcg(reinterpret_cast<const float2*>(W.rpart + rr_ + k));
+            const int xi = __float_as_int(x.y);
+            if (x.x < key || (x.x == key && xi < idx)) {
+              key = x.x;
+              idx = xi;
+            }
           }
-          float km = key;
-#pragma unroll
-          for (int o = 16; o; o >>= 1) km = fminf(km, __shfl_xor_sync(kFull, km, o));
-          const int im = warp_min_i(key == km ? idx : 0x7FFFFFFF);
+          const float km = warp_min(key);
+          const int im = warp_min_i(key == km ? idx : kIntMax);
           if (lane == 0) {
             W.res_done[b] = 0;
-            a.out_tokens[r] = (im != 0x7FFFFFFF) ? im : __ldcg(W.row_targmax + r);
+            a.out_tokens[r] = (im != kIntMax) ? im : __ldcg(W.row_targmax + r);
           }
         }
         e0 += len;
@@ -873,7 +1113,12 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) 
 template <typename T>
 cudaError_t launch_stream_t(int mode, bool sampled, const StreamArgs& a, int grid, size_t smem,
                             cudaStream_t s) {
-#define CMSD_L(M, S) stream_kernel<T, M, S><<<grid, kThreads, smem, s>>>(a)
+#define CMSD_L(M, S)                                                                          \
+  do {                                                                                        \
+    cudaFuncSetAttribute(stream_kernel<T, M, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                         (int)smem);                                                          \
+    stream_kernel<T, M, S><<<grid, kThreads, smem, s>>>(a);                                   \
+  } while (0)
   if (mode == kModeConf) CMSD_L(kModeConf, false);
   else if (mode == kModeVerify) { if (sampled) CMSD_L(kModeVerify, true); else CMSD_L(kModeVerify, false); }
   else { if (sampled) CMSD_L(kModeFused, true); else CMSD_L(kModeFused, false); }
@@ -883,7 +1128,10 @@ cudaError_t launch_stream_t(int mode, bool sampled, const StreamArgs& a, int gri
 
 template <typename T>
 cudaError_t occupancy_stream_t(int mode, bool sampled, size_t smem, int* nb) {
-#define CMSD_O(M, S) cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, stream_kernel<T, M, S>, kThreads, smem)
+#define CMSD_O(M, S)                                                                            \
+  (cudaFuncSetAttribute(stream_kernel<T, M, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,   \
+                        (int)smem),                                                            \
+   cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, stream_kernel<T, M, S>, kThreads, smem))
   if (mode == kModeConf) return CMSD_O(kModeConf, false);
   if (mode == kModeVerify) return sampled ? CMSD_O(kModeVerify, true) : CMSD_O(kModeVerify, false);
   return sampled ? CMSD_O(kModeFused, true) : CMSD_O(kModeFused, false);
