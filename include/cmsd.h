@@ -120,10 +120,14 @@ int cmsd_confidence(const void* draft_logits, int B, int K, int V, int dtype,
  * conf: float [B][K] device, C_t (e.g. from cmsd_confidence).
  * draft_lse: float [B][K] device, drafter log-sum-exp; required for
  *   CMSD_RULE_SAMPLED (q(draft) = exp(z_draft - lse)), ignored otherwise.
- * seed, iteration key the Philox4x32-10 uniforms (SAMPLED): acceptance uniform
- *   counter (0, b, i, iteration<<2 | 0) word 0, residual uniform for entry v
- *   counter (v>>2, b, n, iteration<<2 | 1) word v&3, key (seed lo, seed hi),
- *   u = (word >> 8) 2^-24.
+ * seed, iteration key the Philox4x32-10 uniforms (SAMPLED), key (seed lo,
+ *   seed hi), u = (word >> 8) 2^-24: acceptance uniform counter
+ *   (0, b, i, iteration<<2 | 0) word 0.  The residual token is drawn by a
+ *   two-level exponential race: group g of the 32 entries 32g .. 32g+31 gets
+ *   uniform counter (g>>2, b, n, iteration<<2 | 2) word g&3 and the group with
+ *   the least -log(1-U_g) / R_g wins (R_g its residual mass); entry v of that
+ *   group gets counter (v>>2, b, n, iteration<<2 | 1) word v&3 and the least
+ *   -log(1-U_v) / r_v wins.  The token's law is r_v / sum(r).
  * Outputs: n_accept [B] (first rejected position, k_row[b] if none);
  *   out_tokens [B][K]: accepted drafts, then the correction at n_accept (when
  *   n_accept < k_row[b]), then -1; accept [B][K] (uint8, 0 beyond k_row) may be

@@ -24,7 +24,8 @@ Steps and where the paper defines them:
   SAMPLED rule      speculative sampling of the works cited in Sec. II
                     ([5], [6]), modulated by tau_t: accept with probability
                     min(1, e^tau * p / q), else draw from the normalised
-                    residual max(0, p - q) with an exponential race.
+                    residual max(0, p - q) with a two-level exponential race
+                    (groups of 32 entries, then entries of the winning group).
 
 Readings where the paper is garbled, silent or self-contradictory (each is
 listed with its reason in the design doc):
@@ -225,34 +226,62 @@ def accept_sampled(zt, zd, tok, tau, u, beta_rank):
     return acc, flagged, p, q
 
 
-def residual_token(zt, zd, U):
-    """Draw from norm(max(0, p - q)) by an exponential race over the uniforms U.
-
-    E_v = -log(1 - U_v); the winner is argmin over r_v > 0 of E_v / r_v (lowest
-    index on ties), which has law r / sum(r).  Returns (token, flagged).
-    """
-    p = softmax(zt)
-    q = softmax(zd)
-    r = np.maximum(0.0, p - q)
-    U = np.asarray(U, dtype=np.float64)
-    E = -np.log1p(-U)
+def _race(keys_E, rates, eps=FLAG_EPS, r_lo=None, r_hi=None):
+    """Exponential race: winner = argmin over rates > 0 of E / rate (lowest index
+    on ties).  Returns (winner or -1, flagged); flagged when the winner could
+    change under the given interval [r_lo, r_hi] of each rate and relative eps
+    on each E."""
+    E = np.asarray(keys_E, dtype=np.float64)
+    r = np.asarray(rates, dtype=np.float64)
     cand = r > 0
     if not np.any(cand):
-        return int(np.argmax(np.asarray(zt, dtype=np.float64))), False   # reading R1
+        return -1, False
     with np.errstate(divide="ignore", invalid="ignore"):
         key = np.where(cand, E / np.where(cand, r, 1.0), np.inf)
     w = int(np.argmin(key))
-    # Flag when the winner could change under relative perturbations of FLAG_EPS
-    # in p_v, q_v and E_v.
-    eps = FLAG_EPS
-    r_hi = np.maximum(0.0, p * (1 + eps) - q * (1 - eps))
-    r_lo_w = max(0.0, p[w] * (1 - eps) - q[w] * (1 + eps))
+    if r_lo is None:
+        return w, False
     with np.errstate(divide="ignore", invalid="ignore"):
         key_lo = np.where(r_hi > 0, E * (1 - eps) / np.where(r_hi > 0, r_hi, 1.0), np.inf)
-    key_hi_w = E[w] * (1 + eps) / r_lo_w if r_lo_w > 0 else np.inf
+    key_hi_w = E[w] * (1 + eps) / r_lo[w] if r_lo[w] > 0 else np.inf
     key_lo[w] = np.inf
-    flagged = bool(key_hi_w >= np.min(key_lo))
-    return w, flagged
+    return w, bool(key_hi_w >= np.min(key_lo))
+
+
+def residual_token(zt, zd, seed, b, n, iteration):
+    """Draw from norm(max(0, p - q)) with a two-level exponential race.
+
+    r_v = max(0, p_v - q_v); the vocabulary is cut into groups of
+    philox.GROUP = 32 consecutive entries with mass R_g = sum of r_v over the
+    group.  Level 1: group g gets E_g = -log(1 - U_g) and the winning group is
+    argmin E_g / R_g (law R_g / R).  Level 2: inside the winning group, entry v
+    gets E_v = -log(1 - U_v) and the token is argmin E_v / r_v (law r_v / R_g).
+    Together the token has law r_v / R, the normalised residual.  Ties go to
+    the lowest index.  Returns (token, flagged); flagged when either level's
+    winner could change under relative perturbations of FLAG_EPS in p, q and
+    the exponentials.
+    """
+    p = softmax(zt)
+    q = softmax(zd)
+    V = p.size
+    r = np.maximum(0.0, p - q)
+    if not np.any(r > 0):
+        return int(np.argmax(np.asarray(zt, dtype=np.float64))), False   # reading R1
+    eps = FLAG_EPS
+    r_hi = np.maximum(0.0, p * (1 + eps) - q * (1 - eps))
+    r_lo = np.maximum(0.0, p * (1 - eps) - q * (1 + eps))
+    G = philox.GROUP
+    ng = (V + G - 1) // G
+    pad = ng * G - V
+    R = np.pad(r, (0, pad)).reshape(ng, G).sum(axis=1)
+    R_hi = np.pad(r_hi, (0, pad)).reshape(ng, G).sum(axis=1)
+    R_lo = np.pad(r_lo, (0, pad)).reshape(ng, G).sum(axis=1)
+    Ug = philox.group_uniforms(seed, b, n, iteration, ng)
+    g, f1 = _race(-np.log1p(-Ug), R, eps, R_lo, R_hi)
+    v0, v1 = g * G, min(V, (g + 1) * G)
+    Uv = philox.residual_uniforms(seed, b, n, iteration, V)[v0:v1]
+    k, f2 = _race(-np.log1p(-Uv), r[v0:v1], eps, r_lo[v0:v1], r_hi[v0:v1])
+    return v0 + k, bool(f1 or f2)
 
 
 # ---------------------------------------------------------------------------
@@ -361,9 +390,7 @@ def verify_sequence(draft_b, target_b, tokens_b, conf_b, k_b, P: Params, seed, b
         if P.rule == "paper":
             out[n] = targmax[n]
         else:
-            V = target_b.shape[-1]
-            U = philox.residual_uniforms(seed, b, n, iteration, V)
-            out[n], rflag = residual_token(target_b[n], draft_b[n], U)
+            out[n], rflag = residual_token(target_b[n], draft_b[n], seed, b, n, iteration)
             tok_flag = tok_flag or rflag
     return {"accept": acc, "acc_flag": aflag, "n_accept": n, "n_flag": n_flag,
             "out_tokens": out, "tok_flag": tok_flag, "target_argmax": targmax}

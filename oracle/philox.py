@@ -14,6 +14,8 @@ the parity test: key = (seed low word, seed high word), counter layout
 
     acceptance  u  : counter (0,      b, i, (iteration << 2) | 0), word 0
     residual    U_v: counter (v >> 2, b, n, (iteration << 2) | 1), word v & 3
+    residual    U_g: counter (g >> 2, b, n, (iteration << 2) | 2), word g & 3
+                     (one draw per group g of GROUP = 32 vocabulary entries)
 
 and a 24-bit uniform u = (word >> 8) * 2**-24 in [0, 1), exact in float32.
 
@@ -34,6 +36,8 @@ ROUNDS = 10
 
 PURPOSE_ACCEPT = 0
 PURPOSE_RESIDUAL = 1
+PURPOSE_GROUP = 2
+GROUP = 32
 
 
 def philox4x32_10(counter, key):
@@ -117,4 +121,15 @@ def residual_uniforms(seed, b, n, iteration, V):
     c3 = ((int(iteration) << 2) | PURPOSE_RESIDUAL) & MASK32
     w = philox4x32_10_np(grp, b, n, c3, k0, k1)
     words = np.stack(w, axis=1).reshape(-1)[:V]
+    return word_to_unit(words)
+
+
+def group_uniforms(seed, b, n, iteration, ngroups):
+    """Uniforms U_g, g = 0..ngroups-1, of the group-level residual draw."""
+    k0, k1 = seed_key(seed)
+    nblk = (ngroups + 3) // 4
+    blk = np.arange(nblk, dtype=np.uint64)
+    c3 = ((int(iteration) << 2) | PURPOSE_GROUP) & MASK32
+    w = philox4x32_10_np(blk, b, n, c3, k0, k1)
+    words = np.stack(w, axis=1).reshape(-1)[:ngroups]
     return word_to_unit(words)

@@ -45,8 +45,8 @@ struct __align__(16) Partial {
 };
 
 struct __align__(8) RacePartial {
-  float key;
-  int idx;
+  float key;   // least E_g / R_g of the warp's groups of one row
+  int idx;     // its group (lowest on ties)
 };
 
 struct Workspace {

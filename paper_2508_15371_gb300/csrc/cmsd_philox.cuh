@@ -7,8 +7,8 @@
 // Weyl increments between rounds.
 //
 // The paper (arXiv 2508.15371) does not say how its random draws are made;
-// the acceptance uniform and the residual uniforms use the counter layout
-// documented in include/cmsd.h.
+// the acceptance uniform and the residual (group and entry) uniforms use the
+// counter layout documented in include/cmsd.h.
 #pragma once
 #include <stdint.h>
 
@@ -27,6 +27,7 @@ constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
 
 constexpr uint32_t kPurposeAccept = 0u;
 constexpr uint32_t kPurposeResidual = 1u;
+constexpr uint32_t kPurposeGroup = 2u;
 
 struct U4 { uint32_t x, y, z, w; };
 

@@ -900,200 +900,182 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
 }
 
 // ---------------------------------------------------------------------------
-// residual draw: exponential race over max(0, p - q) at each rejected position
+// residual draw at each rejected position: two-level exponential race over
+// r_v = max(0, p_v - q_v).  Level 1 races the groups of kGroup consecutive
+// entries on their masses R_g = sum of r_v (key E_g / R_g, E_g = -log(1-U_g));
+// level 2 races the entries of the winning group (key E_v / r_v).  The group
+// wins with probability R_g / R and the entry within it with r_v / R_g, so the
+// token has the law r_v / R of the normalised residual.
+//
+// Work is split over warps in units of (rejected row, group); a warp walks its
+// groups GPI at a time, LPG lanes per group with one 16-byte vector each.
+// Its best (key, group) goes to a partial slot; the warp that completes a row
+// merges the partials and runs level 2 on the winning group (one lane per
+// entry).
 // ---------------------------------------------------------------------------
 
-struct Race {
-  float key;
-  int idx;
-  uint32_t grp;
-  U4 words;
+constexpr int kGroup = 32;
+constexpr int kGroupBatch = 128;       // groups whose E_g one warp draws at once (4 per lane)
+constexpr int kResMinGroups = 32;      // fewest groups per warp
+
+struct RowStat {
+  float MLt, invSt, MLd, invSd;
 };
 
-__device__ __forceinline__ uint32_t pick(const U4& w, uint32_t sel) {
-  return sel == 0 ? w.x : sel == 1 ? w.y : sel == 2 ? w.z : w.w;
+// r = max(0, p - q) with every operation rounded on its own, so that level 1
+// and level 2 obtain the same value for the same entry.
+__device__ __forceinline__ float resid(float zt, float zd, const RowStat& s) {
+  const float p = __fmul_rn(ex2(__fmaf_rn(zt, kLog2e, -s.MLt)), s.invSt);
+  const float q = __fmul_rn(ex2(__fmaf_rn(zd, kLog2e, -s.MLd)), s.invSd);
+  return fmaxf(__fsub_rn(p, q), 0.f);
 }
 
-// One candidate of the race: r = p - q; if r > 0 its key is E / r with
-// E = -log(1 - u).  E >= u, so entries with u >= key * r cannot beat the
-// current best and skip the logarithm.
-__device__ __forceinline__ void race_try(Race& rc, float p, float q, uint32_t word, int v) {
-  const float rr = p - q;
-  if (rr > 0.f) {
-    const float u = word_to_unit(word);
-    if (u < rc.key * rr) {
-      const float key = -log1pf(-u) / rr;
-      if (key < rc.key) {
-        rc.key = key;
-        rc.idx = v;
-      }
-    }
-  }
-}
+__device__ __forceinline__ float expo(uint32_t word) { return -log1pf(-word_to_unit(word)); }
 
-// Element-at-a-time form (row heads/tails, and rows whose vectors do not start
-// on a multiple of 4): the Philox block of group v >> 2 is cached per lane.
-__device__ __forceinline__ void race_elem(Race& rc, float zt, float zd, int v, float MLt, float invSt,
-                                          float MLd, float invSd, uint32_t b, uint32_t n,
-                                          uint32_t cw, uint32_t k0, uint32_t k1) {
-  const float p = ex2(fmaf(zt, kLog2e, -MLt)) * invSt;
-  const float q = ex2(fmaf(zd, kLog2e, -MLd)) * invSd;
-  if (p > q) {
-    const uint32_t g = (uint32_t)v >> 2;
-    if (g != rc.grp) {
-      rc.words = philox4x32_10(U4{g, b, n, cw}, k0, k1);
-      rc.grp = g;
-    }
-    race_try(rc, p, q, pick(rc.words, (uint32_t)v & 3u), v);
-  }
-}
-
-// Four consecutive entries v .. v+3 (v a multiple of 4): one Philox block,
-// generated only when some entry of the group has p > q.
-__device__ __forceinline__ void race_group(Race& rc, const float (&zt)[4], const float (&zd)[4], int v,
-                                           float MLt, float invSt, float MLd, float invSd, uint32_t b,
-                                           uint32_t n, uint32_t cw, uint32_t k0, uint32_t k1) {
-  float p[4], q[4];
-  bool any = false;
+template <typename T>
+__device__ __forceinline__ float resid_vec(uint4 qt, uint4 qd, const RowStat& s) {
+  float acc = 0.f;
+  if (sizeof(T) == 2) {
+    const uint32_t wt[4] = {qt.x, qt.y, qt.z, qt.w};
+    const uint32_t wd[4] = {qd.x, qd.y, qd.z, qd.w};
 #pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    p[k] = ex2(fmaf(zt[k], kLog2e, -MLt)) * invSt;
-    q[k] = ex2(fmaf(zd[k], kLog2e, -MLd)) * invSd;
-    any |= p[k] > q[k];
+    for (int k = 0; k < 4; ++k) {
+      acc += resid(bf_lo(wt[k]), bf_lo(wd[k]), s);
+      acc += resid(bf_hi(wt[k]), bf_hi(wd[k]), s);
+    }
+  } else {
+    acc += resid(__uint_as_float(qt.x), __uint_as_float(qd.x), s);
+    acc += resid(__uint_as_float(qt.y), __uint_as_float(qd.y), s);
+    acc += resid(__uint_as_float(qt.z), __uint_as_float(qd.z), s);
+    acc += resid(__uint_as_float(qt.w), __uint_as_float(qd.w), s);
   }
-  if (any) {
-    const U4 rw = philox4x32_10(U4{(uint32_t)v >> 2, b, n, cw}, k0, k1);
-    race_try(rc, p[0], q[0], rw.x, v);
-    race_try(rc, p[1], q[1], rw.y, v + 1);
-    race_try(rc, p[2], q[2], rw.z, v + 2);
-    race_try(rc, p[3], q[3], rw.w, v + 3);
-  }
+  return acc;
 }
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) {
   constexpr int VEC = Elem<T>::kVec;
+  constexpr int LPG = kGroup / VEC;    // lanes per group
+  constexpr int GPI = 32 / LPG;        // groups per warp iteration
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const Workspace& W = a.ws;
   int R = __ldcg(W.rej_count);
   R = R < 0 ? 0 : (R > a.B ? a.B : R);
-  const int64_t N = (int64_t)R * a.V;
-  if (N > 0) {
-    const int Weff = eff_warps(N, 1024, a.nwarps);
+  const int ng = (a.V + kGroup - 1) / kGroup;
+  const int64_t NU = (int64_t)R * ng;
+  if (NU > 0) {
+    const int Weff = eff_warps(NU, kResMinGroups, a.nwarps);
     const int w = blockIdx.x * kWarpsPerBlock + warp;
     if (w < Weff) {
-      int64_t e0 = split_start(w, N, Weff, VEC);
-      const int64_t e1 = split_start(w + 1, N, Weff, VEC);
+      int64_t u0 = split_start(w, NU, Weff, 1);
+      const int64_t u1 = split_start(w + 1, NU, Weff, 1);
       const uint32_t k0 = seed_lo(a.seed), k1 = seed_hi(a.seed);
-      const uint32_t cw = iter_word(a.iteration, kPurposeResidual);
-      while (e0 < e1) {
-        const int rr_ = (int)(e0 / a.V);
-        const int v0 = (int)(e0 - (int64_t)rr_ * a.V);
-        const int len = (int)min((int64_t)(a.V - v0), e1 - e0);
-        const int v1 = v0 + len;
+      const uint32_t cw_grp = iter_word(a.iteration, kPurposeGroup);
+      const int sub = lane % LPG;
+      while (u0 < u1) {
+        const int rr_ = (int)(u0 / ng);
+        const int g0 = (int)(u0 - (int64_t)rr_ * ng);
+        const int cnt = (int)min((int64_t)(ng - g0), u1 - u0);
+        const int g1 = g0 + cnt;
         const int b = __ldcg(W.rej_list + rr_);
         const int n = __ldcg(W.seq_n + b);
         const int r = b * a.K + n;
         const float2 ds = __ldcg(W.row_dstat + r);
         const float2 ts = __ldcg(W.row_tstat + r);
-        const float invSd = 1.0f / ds.y, invSt = 1.0f / ts.y;
+        const RowStat st{ts.x, 1.0f / ts.y, ds.x, 1.0f / ds.y};
         const size_t rowoff = (size_t)r * (size_t)a.V;
         const T* dp = (const T*)a.draft + rowoff;
         const T* tp = (const T*)a.target + rowoff;
+        const bool vec_ok = ((((uintptr_t)tp) | ((uintptr_t)dp)) & 15) == 0;
 
-        Race rc;
-        rc.key = pos_inf();
-        rc.idx = kIntMax;
-        rc.grp = 0xFFFFFFFFu;
-        rc.words = U4{0, 0, 0, 0};
-
-        const int mis = (int)(((uintptr_t)(tp + v0) & 15) / sizeof(T));
-        const int head = mis ? min(VEC - mis, len) : 0;
-        const int va = v0 + head;
-        const int nvec = (v1 - va) / VEC;
-        const int vb = va + nvec * VEC;
-        if (lane < head) {
-          const int v = v0 + lane;
-          race_elem(rc, Elem<T>::load(tp + v), Elem<T>::load(dp + v), v, ts.x, invSt, ds.x, invSd,
-                    b, n, cw, k0, k1);
-        }
-        const uint4* dv = reinterpret_cast<const uint4*>(dp + va);
-        const uint4* tv = reinterpret_cast<const uint4*>(tp + va);
-        if ((va & 3) == 0) {
-          for (int j = lane; j < nvec; j += 32) {
-            const uint4 qd = ld_stream(dv + j), qt = ld_stream(tv + j);
-            const int v = va + j * VEC;
-            if (sizeof(T) == 2) {
-              const float zt0[4] = {bf_lo(qt.x), bf_hi(qt.x), bf_lo(qt.y), bf_hi(qt.y)};
-              const float zd0[4] = {bf_lo(qd.x), bf_hi(qd.x), bf_lo(qd.y), bf_hi(qd.y)};
-              race_group(rc, zt0, zd0, v, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
-              const float zt1[4] = {bf_lo(qt.z), bf_hi(qt.z), bf_lo(qt.w), bf_hi(qt.w)};
-              const float zd1[4] = {bf_lo(qd.z), bf_hi(qd.z), bf_lo(qd.w), bf_hi(qd.w)};
-              race_group(rc, zt1, zd1, v + 4, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
+        float best = pos_inf();
+        int bestg = kIntMax;
+        int gb = -kGroupBatch;               // first group of the drawn batch
+        float E0 = 0.f, E1 = 0.f, E2 = 0.f, E3 = 0.f;
+        for (int gi = g0; gi < g1; gi += GPI) {
+          if (gi + GPI > gb + kGroupBatch) {   // warp-uniform
+            gb = gi & ~3;
+            const U4 wds = philox4x32_10(U4{(uint32_t)(gb >> 2) + (uint32_t)lane, (uint32_t)b,
+                                            (uint32_t)n, cw_grp}, k0, k1);
+            E0 = expo(wds.x); E1 = expo(wds.y); E2 = expo(wds.z); E3 = expo(wds.w);
+          }
+          const int g = gi + lane / LPG;
+          const int v = g * kGroup + sub * VEC;
+          float acc = 0.f;
+          if (g < g1) {
+            if (vec_ok && v + VEC <= a.V) {
+              const uint4 qt = ld_stream(tp + v), qd = ld_stream(dp + v);
+              acc = resid_vec<T>(qt, qd, st);
             } else {
-              const float zt[4] = {__uint_as_float(qt.x), __uint_as_float(qt.y), __uint_as_float(qt.z),
-                                   __uint_as_float(qt.w)};
-              const float zd[4] = {__uint_as_float(qd.x), __uint_as_float(qd.y), __uint_as_float(qd.z),
-                                   __uint_as_float(qd.w)};
-              race_group(rc, zt, zd, v, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
+              for (int k = 0; k < VEC && v + k < a.V; ++k)
+                acc += resid(Elem<T>::load(tp + v + k), Elem<T>::load(dp + v + k), st);
             }
           }
-        } else {
-          for (int j = lane; j < nvec; j += 32) {
-            const uint4 qd = ld_stream(dv + j), qt = ld_stream(tv + j);
-            const int v = va + j * VEC;
-            const uint32_t wd[4] = {qd.x, qd.y, qd.z, qd.w};
-            const uint32_t wt[4] = {qt.x, qt.y, qt.z, qt.w};
-            if (sizeof(T) == 2) {
 #pragma unroll
-              for (int k = 0; k < 4; ++k) {
-                race_elem(rc, bf_lo(wt[k]), bf_lo(wd[k]), v + 2 * k, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
-                race_elem(rc, bf_hi(wt[k]), bf_hi(wd[k]), v + 2 * k + 1, ts.x, invSt, ds.x, invSd, b, n, cw, k0, k1);
-              }
-            } else {
-#pragma unroll
-              for (int k = 0; k < 4; ++k)
-                race_elem(rc, __uint_as_float(wt[k]), __uint_as_float(wd[k]), v + k, ts.x, invSt, ds.x,
-                          invSd, b, n, cw, k0, k1);
+          for (int o = 1; o < LPG; o <<= 1) acc += __shfl_xor_sync(kFull, acc, o);
+          const int off = min(g - gb, kGroupBatch - 1);
+          const int src = off >> 2, sel = off & 3;
+          const float x0 = __shfl_sync(kFull, E0, src), x1 = __shfl_sync(kFull, E1, src);
+          const float x2 = __shfl_sync(kFull, E2, src), x3 = __shfl_sync(kFull, E3, src);
+          const float E = sel == 0 ? x0 : sel == 1 ? x1 : sel == 2 ? x2 : x3;
+          if (g < g1 && acc > 0.f) {
+            const float key = E / acc;
+            if (key < best) {          // groups are visited in increasing order
+              best = key;
+              bestg = g;
             }
           }
         }
-        if (lane < v1 - vb) {
-          const int v = vb + lane;
-          race_elem(rc, Elem<T>::load(tp + v), Elem<T>::load(dp + v), v, ts.x, invSt, ds.x, invSd,
-                    b, n, cw, k0, k1);
-        }
-        // warp: smallest key, lowest index among equal keys
-        const float kmin = warp_min(rc.key);
-        const int imin = warp_min_i(rc.key == kmin ? rc.idx : kIntMax);
-        if (lane == 0) W.rpart[rr_ + w] = RacePartial{kmin, imin};
+        // warp: smallest key, lowest group among equal keys
+        const float kmin = warp_min(best);
+        const int gmin = warp_min_i(best == kmin ? bestg : kIntMax);
+        if (lane == 0) W.rpart[rr_ + w] = RacePartial{kmin, gmin};
         __threadfence();
         int old = 0;
-        if (lane == 0) old = atomicAdd(W.res_done + b, len);
+        if (lane == 0) old = atomicAdd(W.res_done + b, cnt);
         old = __shfl_sync(kFull, old, 0);
-        if (old + len == a.V) {
+        if (old + cnt == ng) {
           __threadfence();
-          const int wf = find_warp((int64_t)rr_ * a.V, N, Weff, VEC);
-          const int wl = find_warp((int64_t)rr_ * a.V + a.V - 1, N, Weff, VEC);
+          const int wf = find_warp((int64_t)rr_ * ng, NU, Weff, 1);
+          const int wl = find_warp((int64_t)rr_ * ng + ng - 1, NU, Weff, 1);
           float key = pos_inf();
-          int idx = kIntMax;
+          int gw = kIntMax;
           for (int k = wf + lane; k <= wl; k += 32) {
             const float2 x = __ldcg(reinterpret_cast<const float2*>(W.rpart + rr_ + k));
-            const int xi = __float_as_int(x.y);
-            if (x.x < key || (x.x == key && xi < idx)) {
+            const int xg = __float_as_int(x.y);
+            if (x.x < key || (x.x == key && xg < gw)) {
               key = x.x;
-              idx = xi;
+              gw = xg;
             }
           }
           const float km = warp_min(key);
-          const int im = warp_min_i(key == km ? idx : kIntMax);
+          const int gm = warp_min_i(key == km ? gw : kIntMax);
+          int tok;
+          if (gm == kIntMax) {
+            tok = __ldcg(W.row_targmax + r);   // empty residual: verifier argmax
+          } else {
+            // level 2: one lane per entry of the winning group
+            const int v = gm * kGroup + lane;
+            float k2 = pos_inf();
+            if (v < a.V) {
+              const float rv = resid(Elem<T>::load(tp + v), Elem<T>::load(dp + v), st);
+              const U4 wds = philox4x32_10(U4{(uint32_t)v >> 2, (uint32_t)b, (uint32_t)n,
+                                              iter_word(a.iteration, kPurposeResidual)}, k0, k1);
+              const uint32_t sel = (uint32_t)v & 3u;
+              const uint32_t word = sel == 0 ? wds.x : sel == 1 ? wds.y : sel == 2 ? wds.z : wds.w;
+              if (rv > 0.f) k2 = expo(word) / rv;
+            }
+            const float k2m = warp_min(k2);
+            const int vm = warp_min_i(k2 == k2m ? v : kIntMax);
+            tok = (vm != kIntMax && k2m != pos_inf()) ? vm : __ldcg(W.row_targmax + r);
+          }
           if (lane == 0) {
             W.res_done[b] = 0;
-            a.out_tokens[r] = (im != kIntMax) ? im : __ldcg(W.row_targmax + r);
+            a.out_tokens[r] = tok;
           }
         }
-        e0 += len;
+        u0 += cnt;
       }
     }
   }

@@ -284,8 +284,7 @@ def test_residual_race_law():
     n = 6000
     counts = np.zeros(8)
     for it in range(n):
-        U = O.philox.residual_uniforms(123, 0, 0, it, 8)
-        tok, _ = O.residual_token(zt, zd, U)
+        tok, _ = O.residual_token(zt, zd, 123, 0, 0, it)
         counts[tok] += 1
     assert counts[r == 0].sum() == 0
     exp = r / r.sum() * n
@@ -346,9 +345,36 @@ def test_sampled_flags_near_threshold():
     assert acc and not flag
 
 
+def test_residual_race_law_across_groups():
+    # V = 100 spans four groups of 32 (the last one partial): the two-level
+    # race must still give each entry probability r_v / sum(r)
+    rng = np.random.default_rng(19)
+    V = 100
+    zt = rng.normal(0, 1.0, V)
+    zd = zt + rng.normal(0, 1.0, V)
+    p, q = sps.softmax(zt), sps.softmax(zd)
+    r = np.maximum(0, p - q)
+    n = 20000
+    counts = np.zeros(V)
+    for it in range(n):
+        tok, _ = O.residual_token(zt, zd, 7, 1, 2, it)
+        counts[tok] += 1
+    assert counts[r == 0].sum() == 0
+    # compare group masses (enough counts per cell) and the within-group law
+    G = O.philox.GROUP
+    gm = np.array([r[i:i + G].sum() for i in range(0, V, G)]) / r.sum() * n
+    gc = np.array([counts[i:i + G].sum() for i in range(0, V, G)])
+    chi2 = ((gc - gm) ** 2 / gm).sum()
+    assert st.chi2.sf(chi2, len(gm) - 1) > 1e-3
+    top = np.argsort(-r)[:8]
+    e = r[top] / r.sum() * n
+    chi2 = ((counts[top] - e) ** 2 / e).sum()
+    assert st.chi2.sf(chi2, len(top)) > 1e-4
+
+
 def test_residual_falls_back_to_target_argmax_when_empty():
     z = np.array([0.1, 2.0, -1.0, 0.5])
-    tok, flag = O.residual_token(z, z, np.full(4, 0.5))
+    tok, flag = O.residual_token(z, z, 0, 0, 0, 0)
     assert tok == 1 and not flag
 
 

@@ -95,6 +95,9 @@ def test_uniforms_are_uniform_and_distinct_streams():
     assert st.pearsonr(U, U2)[0] < 0.01
     acc = np.array([philox.accept_uniform(0, b, i, it) for b in range(8) for i in range(8) for it in range(40)])
     assert st.kstest(acc, "uniform").pvalue > 1e-3
-    # the acceptance stream and the residual stream use different counters
+    # the acceptance, residual-entry and residual-group streams use different counters
     a0 = philox.accept_uniform(5, 3, 2, 9)
     assert a0 != U[0] or a0 != U[1]
+    Ug = philox.group_uniforms(5, 3, 2, 9, 64)
+    assert not np.array_equal(Ug[:8], U[:8])
+    assert st.kstest(philox.group_uniforms(1, 0, 0, 3, 100000), "uniform").pvalue > 1e-3
