@@ -49,7 +49,8 @@ typedef enum {
   CMSD_EDTYPE = -2,     /* unknown dtype or rule */
   CMSD_ECUDA = -3,      /* a CUDA runtime call failed (see cmsd_last_cuda_error) */
   CMSD_ENOWS = -4,      /* workspace NULL or smaller than cmsd_workspace_bytes */
-  CMSD_EALIGN = -5      /* logit base pointer not 16-byte aligned */
+  CMSD_EALIGN = -5,     /* logit base pointer not 16-byte aligned */
+  CMSD_ESCRATCH = -6    /* problem needs more than CMSD_STATIC_SCRATCH_BYTES of scratch */
 } cmsd_status;
 
 typedef enum { CMSD_F32 = 0, CMSD_BF16 = 1 } cmsd_dtype;
@@ -154,6 +155,39 @@ int cmsd_confidence_verify(const void* draft_logits, const void* target_logits,
                            float* H, float* margin, int32_t* argmax, float* conf, float* lse,
                            int32_t* k_next, int32_t* n_accept, int32_t* out_tokens,
                            uint8_t* accept, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * cmsd_confidence_verify without a workspace argument: the scratch is a fixed
+ * array of CMSD_STATIC_SCRATCH_BYTES in the library's device image, one per
+ * device.  This entry point has no counterpart in the paper; it exists for
+ * callers that may not allocate device memory at call time -- e.g. a serving
+ * loop that divides all of HBM once at start-up and treats any later
+ * allocation as an error, or a C caller with no device allocator of its own.
+ * It allocates nothing.
+ *   - Arguments and outputs: as cmsd_confidence_verify, minus ws / ws_bytes.
+ *   - Limit: a problem whose cmsd_workspace_bytes(B, K, V) exceeds
+ *     CMSD_STATIC_SCRATCH_BYTES (4 MiB; on a 152-SM GB300 that admits B*K up
+ *     to about 44,000 positions for K >= 8, 35,000 at K = 1) is rejected with
+ *     CMSD_ESCRATCH before anything is enqueued.
+ *   - Each call first zero-fills, on `stream`, the part of the scratch that
+ *     its layout uses, so device-side error flags (cmsd_workspace_errors) of
+ *     an earlier call are not kept; use cmsd_confidence_verify with a caller
+ *     workspace to read them.
+ *   - One scratch per device: calls whose execution overlaps on one device
+ *     (different streams, or host threads without ordering) race on it and
+ *     give wrong results.  Order all such calls on one stream.
+ *   - The first call on each device does a one-time set-up (it looks up the
+ *     scratch's device address, which may load the module); make that first
+ *     call before any stream capture begins.
+ */
+#define CMSD_STATIC_SCRATCH_BYTES (4u << 20)
+int cmsd_confidence_verify_static(const void* draft_logits, const void* target_logits,
+                                  const int32_t* draft_tokens, const int32_t* k_row,
+                                  int B, int K, int V, int dtype, const cmsd_params* p,
+                                  uint64_t seed, uint32_t iteration,
+                                  float* H, float* margin, int32_t* argmax, float* conf,
+                                  float* lse, int32_t* k_next, int32_t* n_accept,
+                                  int32_t* out_tokens, uint8_t* accept, void* stream);
 
 /* Host-side Philox4x32-10 (the generator the kernels use), for tests:
  * returns output word `word` (0..3) of counter (c0, c1, c2, c3) under key

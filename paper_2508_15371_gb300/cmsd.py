@@ -18,7 +18,7 @@ LIB_PATH = os.path.join(_PKG, "libcmsd.so")
 
 F32, BF16 = 0, 1
 RULE_PAPER, RULE_SAMPLED = 0, 1
-OK, EINVAL, EDTYPE, ECUDA, ENOWS, EALIGN = 0, -1, -2, -3, -4, -5
+OK, EINVAL, EDTYPE, ECUDA, ENOWS, EALIGN, ESCRATCH = 0, -1, -2, -3, -4, -5, -6
 
 _c_int, _c_u32, _c_u64, _c_sz, _vp = ctypes.c_int, ctypes.c_uint32, ctypes.c_uint64, ctypes.c_size_t, ctypes.c_void_p
 
@@ -63,6 +63,9 @@ _SIGS = {
     "cmsd_confidence_verify": (_c_int, [_vp, _vp, _vp, _vp, _c_int, _c_int, _c_int, _c_int, _vp,
                                         _c_u64, _c_u32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                         _vp, _c_sz, _vp]),
+    "cmsd_confidence_verify_static": (_c_int, [_vp, _vp, _vp, _vp, _c_int, _c_int, _c_int, _c_int, _vp,
+                                               _c_u64, _c_u32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                               _vp, _vp]),
     "cmsd_philox_u32": (_c_u32, [_c_u64, _c_u32, _c_u32, _c_u32, _c_u32, _c_int]),
     "cmsd_philox_fill": (_c_int, [_c_u64, _c_u32, _c_u32, _c_u32, _c_u32, _vp, _c_sz, _vp]),
     "cmsd_profile_start": (_c_int, [_c_int]),
@@ -251,6 +254,36 @@ def confidence_verify(draft, target, tokens, k_row=None, p=None, seed=0, iterati
         _ptr(o["conf"]), _ptr(o["lse"]), _ptr(o["k_next"]), _ptr(o["n_accept"]), _ptr(o["out_tokens"]),
         _ptr(o["accept"]), _ptr(ws), ws.numel(), _stream())
     _check(rc, "cmsd_confidence_verify")
+    return o
+
+
+def confidence_verify_static(draft, target, tokens, k_row=None, p=None, seed=0, iteration=0, out=None,
+                             signals=True):
+    """The fused pass through cmsd_confidence_verify_static: the library's own
+    fixed device scratch instead of a workspace (nothing is allocated for it).
+    Output tensors are allocated here unless passed in `out`; a caller that may
+    not allocate passes them all.  Calls on one device must not overlap."""
+    torch = _torch()
+    _need_cuda(draft, target, tokens, k_row)
+    if draft.dtype != target.dtype or draft.shape != target.shape:
+        raise CmsdError("draft and target logits must have the same shape and dtype")
+    B, K, V = draft.shape
+    p = p if p is not None else params(K)
+    dev = draft.device
+    o = {}
+    for n in ("H", "margin", "conf", "lse"):
+        o[n] = _out(out, n, (B, K), torch.float32, dev, signals)
+    o["argmax"] = _out(out, "argmax", (B, K), torch.int32, dev, signals)
+    o["k_next"] = _out(out, "k_next", (B,), torch.int32, dev)
+    o["n_accept"] = _out(out, "n_accept", (B,), torch.int32, dev)
+    o["out_tokens"] = _out(out, "out_tokens", (B, K), torch.int32, dev)
+    o["accept"] = _out(out, "accept", (B, K), torch.uint8, dev, signals)
+    rc = lib().cmsd_confidence_verify_static(
+        _ptr(draft), _ptr(target), _ptr(tokens), _ptr(k_row), B, K, V, _dtype_code(draft),
+        ctypes.byref(p), int(seed), int(iteration), _ptr(o["H"]), _ptr(o["margin"]), _ptr(o["argmax"]),
+        _ptr(o["conf"]), _ptr(o["lse"]), _ptr(o["k_next"]), _ptr(o["n_accept"]), _ptr(o["out_tokens"]),
+        _ptr(o["accept"]), _stream())
+    _check(rc, "cmsd_confidence_verify_static")
     return o
 
 

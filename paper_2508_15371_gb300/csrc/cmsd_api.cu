@@ -441,6 +441,7 @@ const char* cmsd_strerror(int code) {
     case CMSD_ECUDA: return "CUDA runtime error";
     case CMSD_ENOWS: return "workspace missing or too small";
     case CMSD_EALIGN: return "logit pointer not 16-byte aligned";
+    case CMSD_ESCRATCH: return "problem too large for the static scratch (CMSD_STATIC_SCRATCH_BYTES)";
     default: return "unknown error";
   }
 }
