@@ -48,12 +48,27 @@ def peaks():
         return 6800.0, "fallback"
 
 
+KERNEL_SOURCES = ("cmsd_stream_impl.cuh", "cmsd_device.cuh", "cmsd_internal.h")
+
+
+def kernel_sources_sha():
+    import hashlib
+    h = hashlib.sha256()
+    for n in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2508_15371_gb300", "csrc", n), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
 def ncu_traffic():
-    """Per-launch DRAM bytes of the streaming kernel from the committed ncu summary."""
+    """Per-launch DRAM bytes of the streaming kernel from the committed ncu
+    summary; None when the kernel sources changed since it was captured."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             d = json.load(f)
+        if d.get("sources_sha256_16") != kernel_sources_sha():
+            return None
         return d
     except Exception:
         return None
