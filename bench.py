@@ -122,10 +122,31 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(win), "window": note}
 
 
-def make_sets(rank, nsets=2):
+def shard_seeds(rank, nsets=2):
+    """Seeds of the input sets of one rank: every rank gets its own sequences."""
     from paper_2508_15371_gb300 import workloads as W
     base = W.FULL_SIZES[WORKLOAD]["seed"]
-    return [W.make(WORKLOAD, seed=base + 1000 * rank + 100 * j) for j in range(nsets)]
+    return [base + 1000 * rank + 100 * j for j in range(nsets)]
+
+
+def make_sets(rank, nsets=2):
+    from paper_2508_15371_gb300 import workloads as W
+    return [W.make(WORKLOAD, seed=s) for s in shard_seeds(rank, nsets)]
+
+
+def max_over_ranks(ms, dist, device):
+    """The slowest rank's time (ms); every rank gets the same value."""
+    if dist is None:
+        return float(ms)
+    import torch
+    tt = torch.tensor([float(ms)], device=device, dtype=torch.float64)
+    dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+    return float(tt.item())
+
+
+def job_rows_per_s(world, rows_per_rank, steps, ms_total):
+    """Whole-job throughput: the rows all ranks processed over the slowest rank's time."""
+    return world * rows_per_rank * steps / (ms_total * 1e-3)
 
 
 def oracle_rows_per_s(w, p_dict, budget_s, seeds_from=0, max_rows=None):
@@ -270,12 +291,9 @@ def run_ours(args):
     k_ms, r_ms = cmsd.profile_stop(args.steps)
     clocks.stop()
     clk = clocks.summary(t_wall0, t_wall1)
-    if dist:
-        tt = torch.tensor([ms_total], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = max_over_ranks(ms_total, dist, dev)
     ms_step = ms_total / args.steps
-    value = world * rows * args.steps / (ms_total * 1e-3)
+    value = job_rows_per_s(world, rows, args.steps, ms_total)
 
     # ---- end to end: pinned host inputs, copies inside the timed region ----
     e2e_steps = max(3, min(args.steps, 20))
@@ -316,11 +334,8 @@ def run_ours(args):
     e1.record()
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
-    if dist:
-        tt = torch.tensor([e2e_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
-    e2e_value = world * rows * e2e_steps / (e2e_ms * 1e-3)
+    e2e_ms = max_over_ranks(e2e_ms, dist, dev)
+    e2e_value = job_rows_per_s(world, rows, e2e_steps, e2e_ms)
 
     # ---- roofline of the streaming kernel ----------------------------------
     peak, peak_src = peaks()
