@@ -167,7 +167,7 @@ int cmsd_confidence_verify(const void* draft_logits, const void* target_logits,
  *   - Arguments and outputs: as cmsd_confidence_verify, minus ws / ws_bytes.
  *   - Limit: a problem whose cmsd_workspace_bytes(B, K, V) exceeds
  *     CMSD_STATIC_SCRATCH_BYTES (4 MiB; on a 152-SM GB300 that admits B*K up
- *     to about 44,000 positions for K >= 8, 35,000 at K = 1) is rejected with
+ *     to about 41,000 positions for K >= 8, 26,000 at K = 1) is rejected with
  *     CMSD_ESCRATCH before anything is enqueued.
  *   - Each call first zero-fills, on `stream`, the part of the scratch that
  *     its layout uses, so device-side error flags (cmsd_workspace_errors) of

@@ -93,7 +93,7 @@ size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
   size_t err, row_done, seq_done, res_done, rej_count, res_cta_done;
-  size_t rej_list, seq_n, row_conf, row_acc, row_targmax, row_dstat, row_tstat, part, rpart;
+  size_t rej, row_conf, row_acc, row_targmax, row_dstat, row_tstat, part, rpart;
   size_t total;
 };
 
@@ -108,8 +108,7 @@ Layout make_layout(int B, int K, int wmax) {
   L.res_done = o; o += up((size_t)B * sizeof(int));
   L.rej_count = o; o += up(sizeof(int));
   L.res_cta_done = o; o += up(sizeof(int));
-  L.rej_list = o; o += up((size_t)B * sizeof(int));
-  L.seq_n = o; o += up((size_t)B * sizeof(int));
+  L.rej = o; o += up((size_t)B * sizeof(RejRec));
   L.row_conf = o; o += up(BK * sizeof(float));
   L.row_acc = o; o += up(BK * sizeof(int));
   L.row_targmax = o; o += up(BK * sizeof(int));
@@ -130,8 +129,7 @@ Workspace carve(void* ws, const Layout& L) {
   W.res_done = (int*)(p + L.res_done);
   W.rej_count = (int*)(p + L.rej_count);
   W.res_cta_done = (int*)(p + L.res_cta_done);
-  W.rej_list = (int*)(p + L.rej_list);
-  W.seq_n = (int*)(p + L.seq_n);
+  W.rej = (RejRec*)(p + L.rej);
   W.row_conf = (float*)(p + L.row_conf);
   W.row_acc = (int*)(p + L.row_acc);
   W.row_targmax = (int*)(p + L.row_targmax);

@@ -44,22 +44,32 @@ struct __align__(16) Partial {
   int pad[3];
 };
 
-struct __align__(8) RacePartial {
+struct __align__(16) RacePartial {
   float key;   // least E_g / R_g of the warp's groups of one row
-  int idx;     // its group (lowest on ties)
+  int grp;     // its group (lowest on ties)
+  int tok;     // the level-2 winner inside that group
+  int pad;
+};
+
+// One rejected position queued for the residual draw (SAMPLED rule).
+struct __align__(16) RejRec {
+  int r;             // row index b*K + n
+  int b, n;
+  int targmax;       // verifier argmax (fallback for an empty residual)
+  float MLt, invSt;  // verifier: max*log2e, 1 / sum e^(z-max)
+  float MLd, invSd;  // drafter: the same
 };
 
 struct Workspace {
   // counters (zero at rest; each call returns them to zero)
   int* row_done;       // [B*K] logits of the row already reduced
   int* seq_done;       // [B]   rows of the sequence already merged
-  int* res_done;       // [B]   residual-row logits already reduced
+  int* res_done;       // [B]   groups of each queued residual row already raced
   int* rej_count;      // [1]   sequences queued for a residual draw
   int* res_cta_done;   // [1]   CTAs of the resample kernel that finished
   unsigned* err;       // [1]   sticky device-side input errors
   // per-call scratch
-  int* rej_list;       // [B]
-  int* seq_n;          // [B]   first rejected position
+  RejRec* rej;         // [B]   queued rejected positions
   float* row_conf;     // [B*K]
   int* row_acc;        // [B*K]
   int* row_targmax;    // [B*K]

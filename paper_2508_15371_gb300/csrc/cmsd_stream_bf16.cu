@@ -8,8 +8,7 @@ cudaError_t launch_stream_bf16(int mode, bool sampled, const StreamArgs& a, int 
   return launch_stream_t<uint16_t>(mode, sampled, a, grid, smem, s);
 }
 cudaError_t launch_resample_bf16(const StreamArgs& a, int grid, cudaStream_t s) {
-  resample_kernel<uint16_t><<<grid, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  return launch_resample_t<uint16_t>(a, grid, s);
 }
 
 }  // namespace cmsd

@@ -9,8 +9,7 @@ cudaError_t launch_stream_f32(int mode, bool sampled, const StreamArgs& a, int g
   return launch_stream_t<float>(mode, sampled, a, grid, smem, s);
 }
 cudaError_t launch_resample_f32(const StreamArgs& a, int grid, cudaStream_t s) {
-  resample_kernel<float><<<grid, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  return launch_resample_t<float>(a, grid, s);
 }
 
 cudaError_t occupancy_stream(int dtype, int mode, bool sampled, size_t smem, int* nb) {
@@ -18,9 +17,7 @@ cudaError_t occupancy_stream(int dtype, int mode, bool sampled, size_t smem, int
                     : occupancy_stream_t<uint16_t>(mode, sampled, smem, nb);
 }
 cudaError_t occupancy_resample(int dtype, int* nb) {
-  return dtype == 0
-             ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, resample_kernel<float>, kThreads, 0)
-             : cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, resample_kernel<uint16_t>, kThreads, 0);
+  return dtype == 0 ? occupancy_resample_t<float>(nb) : occupancy_resample_t<uint16_t>(nb);
 }
 
 __global__ void philox_fill_kernel(uint32_t k0, uint32_t k1, uint32_t c0, uint32_t c1, uint32_t c2,

@@ -423,6 +423,27 @@ __device__ __forceinline__ int find_warp(int64_t e, int64_t N, int W, int vec) {
   return w;
 }
 
+// a / b for 0 <= a, 0 < b, in 32-bit arithmetic when both fit.
+__device__ __forceinline__ int64_t div_nn(int64_t a, int64_t b) {
+  if (a <= 0x7FFFFFFF && b <= 0x7FFFFFFF) return (int64_t)((uint32_t)a / (uint32_t)b);
+  return a / b;
+}
+
+// N units over W warps, contiguous and in order: the first rem warps get q+1.
+struct EvenSplit {
+  int64_t q;
+  int rem;
+  __device__ EvenSplit(int64_t N, int W) {
+    q = div_nn(N, W);
+    rem = (int)(N - q * W);
+  }
+  __device__ int64_t start(int w) const { return (int64_t)w * q + (w < rem ? w : rem); }
+  __device__ int owner(int64_t u) const {
+    const int64_t big = (q + 1) * rem;
+    return u < big ? (int)div_nn(u, q + 1) : rem + (int)div_nn(u - big, q);
+  }
+};
+
 __device__ __forceinline__ int k_of(const StreamArgs& a, int b) {
   if (!a.k_row) return a.K;
   int k = __ldg(a.k_row + b);
@@ -532,8 +553,15 @@ __device__ void seq_epilogue(const StreamArgs& a, int b, int kb, int lane) {
       if (SAMPLED && n < kb) {
         const int slot = atomicAdd(W.rej_count, 1);
         if (slot < a.B) {
-          W.rej_list[slot] = b;
-          W.seq_n[b] = n;
+          const int r = base + n;
+          const float2 ts = __ldcg(W.row_tstat + r);
+          const float2 ds = __ldcg(W.row_dstat + r);
+          RejRec q;
+          q.r = r; q.b = b; q.n = n;
+          q.targmax = __ldcg(W.row_targmax + r);
+          q.MLt = ts.x; q.invSt = 1.0f / ts.y;
+          q.MLd = ds.x; q.invSd = 1.0f / ds.y;
+          W.rej[slot] = q;
         } else {
           atomicOr(W.err, 4u);   // queue not drained by a previous call: workspace misuse
         }
@@ -830,6 +858,9 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
   constexpr bool HAS_T = MODE != kModeConf;
   constexpr int VEC = Elem<T>::kVec;
   extern __shared__ __align__(128) unsigned char smem[];
+  // the resample kernel (launched as a programmatic dependent) may be
+  // scheduled now; it waits for this grid's completion before reading anything
+  if (SAMPLED) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
@@ -914,51 +945,147 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
 // entry).
 // ---------------------------------------------------------------------------
 
+#ifndef CMSD_RES_MIN_BLOCKS
+#define CMSD_RES_MIN_BLOCKS 3
+#endif
 constexpr int kGroup = 32;
 constexpr int kGroupBatch = 128;       // groups whose E_g one warp draws at once (4 per lane)
-constexpr int kResMinGroups = 32;      // fewest groups per warp
+constexpr int kResMinGroups = 48;      // fewest groups per warp
+constexpr int kResStageBytes = 8192;   // shared-memory stage per warp (both tensors)
+constexpr float kRaceFilter = 0.99999f;  // 1 - 1e-5
 
 struct RowStat {
-  float MLt, invSt, MLd, invSd;
+  float MLt, invSt;    // verifier: max*log2e, 1 / sum
+  float MLd, ninvSd;   // drafter: max*log2e, -1 / sum
 };
 
-// r = max(0, p - q) with every operation rounded on its own, so that level 1
-// and level 2 obtain the same value for the same entry.
+// r = max(0, p - q), p = e^(zt - Mt) / St, q = e^(zd - Md) / Sd, with every
+// operation rounded on its own (p - q formed as p + (-q), which is the same
+// rounding), so that the packed form below gives the same bits per entry.
 __device__ __forceinline__ float resid(float zt, float zd, const RowStat& s) {
   const float p = __fmul_rn(ex2(__fmaf_rn(zt, kLog2e, -s.MLt)), s.invSt);
-  const float q = __fmul_rn(ex2(__fmaf_rn(zd, kLog2e, -s.MLd)), s.invSd);
-  return fmaxf(__fsub_rn(p, q), 0.f);
+  const float qn = __fmul_rn(ex2(__fmaf_rn(zd, kLog2e, -s.MLd)), s.ninvSd);
+  return fmaxf(__fadd_rn(p, qn), 0.f);
 }
 
 __device__ __forceinline__ float expo(uint32_t word) { return -log1pf(-word_to_unit(word)); }
 
+// resid() of two entries at once (packed f32x2), accumulated into acc.
+__device__ __forceinline__ void resid2(u64& acc, u64 zt, u64 zd, const RowStat& s) {
+  const u64 p = mul2(ex2_2(fma2(zt, dup2(kLog2e), dup2(-s.MLt))), dup2(s.invSt));
+  const u64 qn = mul2(ex2_2(fma2(zd, dup2(kLog2e), dup2(-s.MLd))), dup2(s.ninvSd));
+  const u64 r = add2(p, qn);
+  acc = add2(acc, pack2(fmaxf(lo32f(r), 0.f), fmaxf(hi32f(r), 0.f)));
+}
+
+// Sum of r over the entries of one 16-byte vector pair.
 template <typename T>
 __device__ __forceinline__ float resid_vec(uint4 qt, uint4 qd, const RowStat& s) {
-  float acc = 0.f;
+  u64 acc = 0ull;
   if (sizeof(T) == 2) {
-    const uint32_t wt[4] = {qt.x, qt.y, qt.z, qt.w};
-    const uint32_t wd[4] = {qd.x, qd.y, qd.z, qd.w};
+    resid2(acc, bf2_to_f2(qt.x), bf2_to_f2(qd.x), s);
+    resid2(acc, bf2_to_f2(qt.y), bf2_to_f2(qd.y), s);
+    resid2(acc, bf2_to_f2(qt.z), bf2_to_f2(qd.z), s);
+    resid2(acc, bf2_to_f2(qt.w), bf2_to_f2(qd.w), s);
+  } else {
+    resid2(acc, pack2(__uint_as_float(qt.x), __uint_as_float(qt.y)),
+           pack2(__uint_as_float(qd.x), __uint_as_float(qd.y)), s);
+    resid2(acc, pack2(__uint_as_float(qt.z), __uint_as_float(qt.w)),
+           pack2(__uint_as_float(qd.z), __uint_as_float(qd.w)), s);
+  }
+  return lo32f(acc) + hi32f(acc);
+}
+
+// GPU-scope add with acquire-release semantics: the caller's earlier stores
+// are visible before the add, and what other threads released before their
+// adds is visible after it.
+__device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
+  int old;
+  asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
+// 16 bytes of logits at entry v of one row: one vector load when the vector is
+// aligned and inside the row, else element loads with entries past the row
+// end read as -inf (p = q = 0, so r = 0).
+template <typename T>
+__device__ __forceinline__ uint4 load_logits(const T* p, int v, int V, bool vec_ok) {
+  constexpr int VEC = Elem<T>::kVec;
+  if (vec_ok && v + VEC <= V) return ld_stream(p + v);
+  uint32_t w[4];
+  if (sizeof(T) == 2) {
+    const unsigned short* q = reinterpret_cast<const unsigned short*>(p);
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-      acc += resid(bf_lo(wt[k]), bf_lo(wd[k]), s);
-      acc += resid(bf_hi(wt[k]), bf_hi(wd[k]), s);
+      const uint32_t lo = (v + 2 * k < V) ? (uint32_t)__ldg(q + v + 2 * k) : 0xFF80u;
+      const uint32_t hi = (v + 2 * k + 1 < V) ? (uint32_t)__ldg(q + v + 2 * k + 1) : 0xFF80u;
+      w[k] = lo | (hi << 16);
     }
   } else {
-    acc += resid(__uint_as_float(qt.x), __uint_as_float(qd.x), s);
-    acc += resid(__uint_as_float(qt.y), __uint_as_float(qd.y), s);
-    acc += resid(__uint_as_float(qt.z), __uint_as_float(qd.z), s);
-    acc += resid(__uint_as_float(qt.w), __uint_as_float(qd.w), s);
+    const uint32_t* q = reinterpret_cast<const uint32_t*>(p);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) w[k] = (v + k < V) ? __ldg(q + v + k) : 0xFF800000u;
   }
-  return acc;
+  return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
 template <typename T>
-__global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) {
+__device__ __forceinline__ uint4 neg_inf_vec() {
+  return sizeof(T) == 2 ? make_uint4(kNegInf2, kNegInf2, kNegInf2, kNegInf2)
+                        : make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
+}
+
+// Entry k of a 16-byte vector (k may be a run-time value: selects, no local array).
+template <typename T>
+__device__ __forceinline__ float logit_at(uint4 q, int k) {
+  const int j = sizeof(T) == 2 ? (k >> 1) : k;
+  const uint32_t w = j == 0 ? q.x : j == 1 ? q.y : j == 2 ? q.z : q.w;
+  if (sizeof(T) == 2) return (k & 1) ? bf_hi(w) : bf_lo(w);
+  return __uint_as_float(w);
+}
+
+// Level 2 on group gm, whose logits sit in lanes own .. own+LPG-1 (vector
+// `sub` of the group in lane own+sub): every lane takes one entry, gathers its
+// logit pair by shuffles and races E_v / r_v.  Returns the warp's least key
+// (lowest entry on ties) as the entry index, or -1 if no entry has r_v > 0.
+template <typename T>
+__device__ __forceinline__ int race_group_entries(uint4 qt, uint4 qd, int gm, int own, int lane,
+                                                  const RowStat& st, uint32_t b, uint32_t n,
+                                                  uint32_t cw, uint32_t k0, uint32_t k1) {
+  constexpr int VEC = Elem<T>::kVec;
+  const int src = own + lane / VEC;
+  const int k = lane % VEC;
+  const uint32_t t0 = __shfl_sync(kFull, qt.x, src), t1 = __shfl_sync(kFull, qt.y, src);
+  const uint32_t t2 = __shfl_sync(kFull, qt.z, src), t3 = __shfl_sync(kFull, qt.w, src);
+  const uint32_t d0 = __shfl_sync(kFull, qd.x, src), d1 = __shfl_sync(kFull, qd.y, src);
+  const uint32_t d2 = __shfl_sync(kFull, qd.z, src), d3 = __shfl_sync(kFull, qd.w, src);
+  const float zt = logit_at<T>(make_uint4(t0, t1, t2, t3), k);
+  const float zd = logit_at<T>(make_uint4(d0, d1, d2, d3), k);
+  const int v = gm * kGroup + lane;
+  const float rv = resid(zt, zd, st);
+  const U4 wd = philox4x32_10(U4{(uint32_t)v >> 2, b, n, cw}, k0, k1);
+  const uint32_t sel = (uint32_t)v & 3u;
+  const uint32_t word = sel == 0 ? wd.x : sel == 1 ? wd.y : sel == 2 ? wd.z : wd.w;
+  const float key = rv > 0.f ? expo(word) / rv : pos_inf();
+  const float km = warp_min(key);
+  const int vm = warp_min_i(key == km ? v : kIntMax);
+  return km != pos_inf() ? vm : -1;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads, CMSD_RES_MIN_BLOCKS) resample_kernel(const StreamArgs a) {
   constexpr int VEC = Elem<T>::kVec;
   constexpr int LPG = kGroup / VEC;    // lanes per group
   constexpr int GPI = 32 / LPG;        // groups per warp iteration
+  constexpr int CG = kResStageBytes / (2 * kGroup * (int)sizeof(T));   // groups per chunk
+  extern __shared__ __align__(16) unsigned char res_smem[];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
+  const unsigned char* stage = res_smem + warp * kResStageBytes;
+  const uint32_t st_t = smem_u32(stage), st_d = st_t + kResStageBytes / 2;
+  // everything below reads what the streaming kernel wrote: wait until that
+  // grid has completed and its memory is visible
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const Workspace& W = a.ws;
   int R = __ldcg(W.rej_count);
   R = R < 0 ? 0 : (R > a.B ? a.B : R);
@@ -968,111 +1095,130 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) 
     const int Weff = eff_warps(NU, kResMinGroups, a.nwarps);
     const int w = blockIdx.x * kWarpsPerBlock + warp;
     if (w < Weff) {
-      int64_t u0 = split_start(w, NU, Weff, 1);
-      const int64_t u1 = split_start(w + 1, NU, Weff, 1);
+      const EvenSplit sp(NU, Weff);
+      int64_t u0 = sp.start(w);
+      const int64_t u1 = sp.start(w + 1);
       const uint32_t k0 = seed_lo(a.seed), k1 = seed_hi(a.seed);
       const uint32_t cw_grp = iter_word(a.iteration, kPurposeGroup);
+      const uint32_t cw_ent = iter_word(a.iteration, kPurposeResidual);
       const int sub = lane % LPG;
       while (u0 < u1) {
-        const int rr_ = (int)(u0 / ng);
+        const int rr_ = (int)div_nn(u0, ng);
         const int g0 = (int)(u0 - (int64_t)rr_ * ng);
         const int cnt = (int)min((int64_t)(ng - g0), u1 - u0);
         const int g1 = g0 + cnt;
-        const int b = __ldcg(W.rej_list + rr_);
-        const int n = __ldcg(W.seq_n + b);
-        const int r = b * a.K + n;
-        const float2 ds = __ldcg(W.row_dstat + r);
-        const float2 ts = __ldcg(W.row_tstat + r);
-        const RowStat st{ts.x, 1.0f / ts.y, ds.x, 1.0f / ds.y};
+        const int4 rq0 = __ldcg(reinterpret_cast<const int4*>(W.rej + rr_));
+        const float4 rq1 = __ldcg(reinterpret_cast<const float4*>(W.rej + rr_) + 1);
+        const int r = rq0.x, b = rq0.y, n = rq0.z;
+        const RowStat st{rq1.x, rq1.y, rq1.z, -rq1.w};
         const size_t rowoff = (size_t)r * (size_t)a.V;
         const T* dp = (const T*)a.draft + rowoff;
         const T* tp = (const T*)a.target + rowoff;
         const bool vec_ok = ((((uintptr_t)tp) | ((uintptr_t)dp)) & 15) == 0;
 
-        float best = pos_inf();
+        // level 1, one chunk of CG groups at a time: the chunk's logits are
+        // copied to this warp's shared-memory stage in one batch of cp.async
+        // (all in flight together), then raced GPI groups per iteration
+        float best = pos_inf();              // this lane set's least key
+        float thr = pos_inf();               // the warp's least key so far (filter bound)
         int bestg = kIntMax;
+        uint4 bqt = neg_inf_vec<T>(), bqd = neg_inf_vec<T>();
         int gb = -kGroupBatch;               // first group of the drawn batch
-        float E0 = 0.f, E1 = 0.f, E2 = 0.f, E3 = 0.f;
-        for (int gi = g0; gi < g1; gi += GPI) {
-          if (gi + GPI > gb + kGroupBatch) {   // warp-uniform
-            gb = gi & ~3;
-            const U4 wds = philox4x32_10(U4{(uint32_t)(gb >> 2) + (uint32_t)lane, (uint32_t)b,
-                                            (uint32_t)n, cw_grp}, k0, k1);
-            E0 = expo(wds.x); E1 = expo(wds.y); E2 = expo(wds.z); E3 = expo(wds.w);
+        uint32_t U0 = 0, U1 = 0, U2 = 0, U3 = 0;
+        for (int gc = g0; gc < g1; gc += CG) {
+          const int ge = min(g1, gc + CG);
+          const int v_base = gc * kGroup;
+          // vectors of the chunk lying wholly inside the row (aligned rows only)
+          const int nfull = vec_ok ? min((ge - gc) * LPG, (a.V - v_base) / VEC) : 0;
+          for (int j = lane; j < nfull; j += 32) {
+            cp_async16(st_t + 16u * (uint32_t)j, tp + v_base + j * VEC);
+            cp_async16(st_d + 16u * (uint32_t)j, dp + v_base + j * VEC);
           }
-          const int g = gi + lane / LPG;
-          const int v = g * kGroup + sub * VEC;
-          float acc = 0.f;
-          if (g < g1) {
-            if (vec_ok && v + VEC <= a.V) {
-              const uint4 qt = ld_stream(tp + v), qd = ld_stream(dp + v);
-              acc = resid_vec<T>(qt, qd, st);
-            } else {
-              for (int k = 0; k < VEC && v + k < a.V; ++k)
-                acc += resid(Elem<T>::load(tp + v + k), Elem<T>::load(dp + v + k), st);
+          cp_async_commit();
+          cp_async_wait<0>();
+          __syncwarp();
+          for (int gi = gc; gi < ge; gi += GPI) {
+            const int g = gi + lane / LPG;
+            const int j = (g - gc) * LPG + sub;
+            uint4 qt = neg_inf_vec<T>(), qd = neg_inf_vec<T>();
+            if (g < ge) {
+              if (j < nfull) {
+                qt = *reinterpret_cast<const uint4*>(stage + 16 * j);
+                qd = *reinterpret_cast<const uint4*>(stage + kResStageBytes / 2 + 16 * j);
+              } else {   // ragged row end or unaligned row: element loads, -inf past the end
+                qt = load_logits<T>(tp, g * kGroup + sub * VEC, a.V, false);
+                qd = load_logits<T>(dp, g * kGroup + sub * VEC, a.V, false);
+              }
             }
-          }
+            if (gi + GPI > gb + kGroupBatch) {   // warp-uniform
+              gb = gi & ~3;
+              const U4 wds = philox4x32_10(U4{(uint32_t)(gb >> 2) + (uint32_t)lane, (uint32_t)b,
+                                              (uint32_t)n, cw_grp}, k0, k1);
+              U0 = wds.x; U1 = wds.y; U2 = wds.z; U3 = wds.w;
+            }
+            float acc = resid_vec<T>(qt, qd, st);
 #pragma unroll
-          for (int o = 1; o < LPG; o <<= 1) acc += __shfl_xor_sync(kFull, acc, o);
-          const int off = min(g - gb, kGroupBatch - 1);
-          const int src = off >> 2, sel = off & 3;
-          const float x0 = __shfl_sync(kFull, E0, src), x1 = __shfl_sync(kFull, E1, src);
-          const float x2 = __shfl_sync(kFull, E2, src), x3 = __shfl_sync(kFull, E3, src);
-          const float E = sel == 0 ? x0 : sel == 1 ? x1 : sel == 2 ? x2 : x3;
-          if (g < g1 && acc > 0.f) {
-            const float key = E / acc;
-            if (key < best) {          // groups are visited in increasing order
-              best = key;
-              bestg = g;
+            for (int o = 1; o < LPG; o <<= 1) acc += __shfl_xor_sync(kFull, acc, o);
+            const int off = min(g - gb, kGroupBatch - 1);
+            const int src = off >> 2, sel = off & 3;
+            const uint32_t x0 = __shfl_sync(kFull, U0, src), x1 = __shfl_sync(kFull, U1, src);
+            const uint32_t x2 = __shfl_sync(kFull, U2, src), x3 = __shfl_sync(kFull, U3, src);
+            const uint32_t word = sel == 0 ? x0 : sel == 1 ? x1 : sel == 2 ? x2 : x3;
+            // E_g >= U_g, so a group with U_g >= thr * R_g has a key above the
+            // warp's best so far and cannot win (the factor keeps the filter
+            // safe against the rounding of E and of the product)
+            bool improved = false;
+            if (g < ge && acc > 0.f && word_to_unit(word) * kRaceFilter < thr * acc) {
+              const float key = expo(word) / acc;
+              if (key < best) {          // groups are visited in increasing order
+                best = key;
+                bestg = g;
+                bqt = qt;
+                bqd = qd;
+                improved = true;
+              }
             }
+            if (__any_sync(kFull, improved)) thr = warp_min(best);
           }
+          __syncwarp();                  // the stage is rewritten by the next chunk
         }
-        // warp: smallest key, lowest group among equal keys
         const float kmin = warp_min(best);
         const int gmin = warp_min_i(best == kmin ? bestg : kIntMax);
-        if (lane == 0) W.rpart[rr_ + w] = RacePartial{kmin, gmin};
-        __threadfence();
+        // level 2 on this warp's winning group (its lanes are the ones whose
+        // best group it is)
+        int tok = -1;
+        if (gmin != kIntMax) {
+          const int own = ((gmin - g0) % GPI) * LPG;
+          tok = race_group_entries<T>(bqt, bqd, gmin, own, lane, st, (uint32_t)b, (uint32_t)n,
+                                      cw_ent, k0, k1);
+        }
         int old = 0;
-        if (lane == 0) old = atomicAdd(W.res_done + b, cnt);
+        if (lane == 0) {
+          W.rpart[rr_ + w] = RacePartial{kmin, gmin, tok, 0};
+          old = atom_add_acq_rel(W.res_done + rr_, cnt);
+        }
         old = __shfl_sync(kFull, old, 0);
         if (old + cnt == ng) {
-          __threadfence();
-          const int wf = find_warp((int64_t)rr_ * ng, NU, Weff, 1);
-          const int wl = find_warp((int64_t)rr_ * ng + ng - 1, NU, Weff, 1);
+          __syncwarp();
+          const int wf = sp.owner((int64_t)rr_ * ng);
+          const int wl = sp.owner((int64_t)rr_ * ng + ng - 1);
           float key = pos_inf();
-          int gw = kIntMax;
+          int gw = kIntMax, tw = -1;
           for (int k = wf + lane; k <= wl; k += 32) {
-            const float2 x = __ldcg(reinterpret_cast<const float2*>(W.rpart + rr_ + k));
-            const int xg = __float_as_int(x.y);
-            if (x.x < key || (x.x == key && xg < gw)) {
-              key = x.x;
-              gw = xg;
+            const int4 x = __ldcg(reinterpret_cast<const int4*>(W.rpart + rr_ + k));
+            const float xk = __int_as_float(x.x);
+            if (xk < key || (xk == key && x.y < gw)) {
+              key = xk;
+              gw = x.y;
+              tw = x.z;
             }
           }
           const float km = warp_min(key);
           const int gm = warp_min_i(key == km ? gw : kIntMax);
-          int tok;
-          if (gm == kIntMax) {
-            tok = __ldcg(W.row_targmax + r);   // empty residual: verifier argmax
-          } else {
-            // level 2: one lane per entry of the winning group
-            const int v = gm * kGroup + lane;
-            float k2 = pos_inf();
-            if (v < a.V) {
-              const float rv = resid(Elem<T>::load(tp + v), Elem<T>::load(dp + v), st);
-              const U4 wds = philox4x32_10(U4{(uint32_t)v >> 2, (uint32_t)b, (uint32_t)n,
-                                              iter_word(a.iteration, kPurposeResidual)}, k0, k1);
-              const uint32_t sel = (uint32_t)v & 3u;
-              const uint32_t word = sel == 0 ? wds.x : sel == 1 ? wds.y : sel == 2 ? wds.z : wds.w;
-              if (rv > 0.f) k2 = expo(word) / rv;
-            }
-            const float k2m = warp_min(k2);
-            const int vm = warp_min_i(k2 == k2m ? v : kIntMax);
-            tok = (vm != kIntMax && k2m != pos_inf()) ? vm : __ldcg(W.row_targmax + r);
-          }
+          const int tm = warp_min_i((key == km && gw == gm && tw >= 0) ? tw : kIntMax);
           if (lane == 0) {
-            W.res_done[b] = 0;
-            a.out_tokens[r] = tok;
+            W.res_done[rr_] = 0;
+            a.out_tokens[r] = (gm != kIntMax && tm != kIntMax) ? tm : rq0.w;   // empty residual: argmax
           }
         }
         u0 += cnt;
@@ -1082,14 +1228,40 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const StreamArgs a) 
   // the last CTA to finish clears the queue for the next call
   __syncthreads();
   if (threadIdx.x == 0) {
-    __threadfence();
-    const int done = atomicAdd(W.res_cta_done, 1);
+    const int done = atom_add_acq_rel(W.res_cta_done, 1);
     if (done == (int)gridDim.x - 1) {
       *W.rej_count = 0;
       *W.res_cta_done = 0;
       __threadfence();
     }
   }
+}
+
+constexpr size_t kResSmemBytes = (size_t)kWarpsPerBlock * kResStageBytes;
+
+// Launched as a programmatic dependent of the streaming kernel just before it
+// on the same stream: its CTAs may be scheduled as the streaming kernel's CTAs
+// retire, and griddepcontrol.wait at its top orders it after that grid.
+template <typename T>
+cudaError_t launch_resample_t(const StreamArgs& a, int grid, cudaStream_t s) {
+  cudaFuncSetAttribute(resample_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kResSmemBytes);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kResSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, resample_kernel<T>, a);
+}
+
+template <typename T>
+cudaError_t occupancy_resample_t(int* nb) {
+  cudaFuncSetAttribute(resample_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kResSmemBytes);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, resample_kernel<T>, kThreads, kResSmemBytes);
 }
 
 template <typename T>
