@@ -12,23 +12,12 @@ constexpr int kMaxRaggedB = 12000;            // B limit when k_row is given (pr
 
 enum Mode { kModeConf = 0, kModeVerify = 1, kModeFused = 2 };
 
-// Per-warp shared-memory staging of the streaming kernel: kStagesRing stages,
-// each CMSD_UNROLL 16-byte vectors per lane of drafter and of target logits.
-#ifndef CMSD_STAGES
-#define CMSD_STAGES 3
-#endif
-#ifndef CMSD_UNROLL
-#define CMSD_UNROLL 2
-#endif
-constexpr int kStagesRing = CMSD_STAGES;
-constexpr int kStageWarpBytes = CMSD_UNROLL * 2 * 512;   // one stage of one warp
-
-// dynamic shared memory of one CTA: [k_row prefix][per-warp stage rings]
+// dynamic shared memory of one streaming CTA: the k_row prefix (ragged windows)
 __host__ __device__ inline size_t stream_pref_bytes(int B, bool ragged) {
   return ragged ? (((size_t)(B + 1) * sizeof(int) + 127) / 128) * 128 : 0;
 }
 __host__ __device__ inline size_t stream_smem_bytes(int B, bool ragged) {
-  return stream_pref_bytes(B, ragged) + (size_t)kWarpsPerBlock * kStagesRing * kStageWarpBytes;
+  return stream_pref_bytes(B, ragged);
 }
 
 // One warp's reduction over one row segment (or, in the row merge, the

@@ -286,18 +286,32 @@ template <> __device__ __forceinline__ float4 as_vec<float>(uint4 r) {
 }
 template <> __device__ __forceinline__ uint4 as_vec<uint16_t>(uint4 r) { return r; }
 
+// Entry k of a 16-byte vector (k may be a run-time value: selects, no local array).
+template <typename T>
+__device__ __forceinline__ float logit_at(uint4 q, int k) {
+  const int j = sizeof(T) == 2 ? (k >> 1) : k;
+  const uint32_t w = j == 0 ? q.x : j == 1 ? q.y : j == 2 ? q.z : q.w;
+  if (sizeof(T) == 2) return (k & 1) ? bf_hi(w) : bf_lo(w);
+  return __uint_as_float(w);
+}
+
 // First index in the unit (start pos, width w) whose value equals m (drafter
-// values clamped as in the streaming pass when `clamp`).
+// values clamped as in the streaming pass when `clamp`).  A unit of width > 1
+// is one aligned 16-byte vector of the row: it is read with a single load
+// and searched in registers.
 template <typename T>
 __device__ __forceinline__ int first_equal(const T* row, int pos, int w, float m, bool clamp) {
   if (w <= 1) return pos;
+  const uint4 q = __ldcg(reinterpret_cast<const uint4*>(row + pos));
   const float nc = neg_clamp();
-  for (int k = 0; k < w; ++k) {
-    float z = Elem<T>::load(row + pos + k);
+  int k = w;
+#pragma unroll
+  for (int j = Elem<T>::kVec - 1; j >= 0; --j) {
+    float z = logit_at<T>(q, j);
     if (clamp) z = fmaxf(z, nc);
-    if (z == m) return pos + k;
+    k = (z == m) ? j : k;
   }
-  return pos;   // not reached
+  return k < w ? pos + k : pos;
 }
 
 // ---------------------------------------------------------------------------
@@ -641,11 +655,10 @@ __device__ void row_results(const StreamArgs& a, int r, int b, int i, const DRed
 //
 // Every warp owns one contiguous slice of the stream.  Within each segment
 // (the part of one row inside the slice) a lane's 16-byte vectors are those
-// with index lane + 32 t; they are staged kStagesRing stages ahead, CMSD_UNROLL
-// vectors of each tensor per stage, by asynchronous global->shared copies
-// into the lane's own slots, and read back by the same lane, so no lane waits
-// on another and the waits (cp.async.wait_group) block in hardware.  A
-// segment's unaligned head and tail (under 16 bytes each) are read directly.
+// with index lane + 32 t, CMSD_UNROLL of each tensor per stage; the loads of
+// stage s+1 are issued into registers before stage s is reduced, so every
+// lane keeps one stage in flight and no lane waits on another.  A segment's
+// unaligned head and tail (under 16 bytes each) are read directly.
 // At the end of a segment the warp reduces its lanes and writes one Partial;
 // the warp that completes a row merges the row and, when it completes a
 // sequence, runs the sequence epilogue.  Warps never wait on each other.
@@ -760,67 +773,63 @@ __device__ __forceinline__ float target_at_token(const StreamArgs& a, int r) {
 
 // ---- one segment body, pipelined ----------------------------------------------
 // The lane's vectors of the aligned body [va, vb) are j = lane + 32 t,
-// t = 0, 1, ...; stage s holds t in [s*U, s*U + U).  Stages are copied
-// kStagesRing ahead with asynchronous copies into the lane's own slots and
-// read back by the same lane.
+// t = 0, 1, ...; stage s holds t in [s*U, s*U + U) and is loaded (streaming,
+// no L1 allocation) while stage s-1 is reduced.
 #ifndef CMSD_UNROLL
 #define CMSD_UNROLL 2
 #endif
 template <typename T, int MODE, bool SAMPLED>
 __device__ __forceinline__ void walk_body(SegState<T>& ss, const T* dp, const T* tp, int va, int vb, int beta,
-                                          unsigned char* lane_ring, int lane) {
+                                          int lane) {
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   constexpr int VEC = Elem<T>::kVec;
   constexpr int U = CMSD_UNROLL;
-  constexpr int SLOT = U * 2 * 512;                  // bytes of one stage of one warp
   const int nvec = (vb - va) / VEC;
   if (nvec <= 0) return;
-  const int nt = nvec > lane ? (nvec - lane + 31) / 32 : 0;   // this lane's vectors
-  const int nst = (nt + U - 1) / U;                            // this lane's stages
-  const unsigned char* gd = reinterpret_cast<const unsigned char*>(dp + va) + 16 * lane;
-  const unsigned char* gt = HAS_T ? reinterpret_cast<const unsigned char*>(tp + va) + 16 * lane : nullptr;
-  const uint32_t ring_s = smem_u32(lane_ring);
-  // issue stage s (vectors t = s*U + u of this lane) into slot s % kStagesRing
-  auto issue = [&](int s, uint32_t slot_s) {
-    if (s < nst) {
-      const int t0 = s * U;
-      const size_t go = (size_t)t0 * 512;
+  const int nt = nvec > lane ? (nvec - lane + 31) / 32 : 0;
+  const int nst = (nvec + 32 * U - 1) / (32 * U);
+  const uint4* gd = reinterpret_cast<const uint4*>(dp + va) + lane;
+  const uint4* gt = HAS_T ? reinterpret_cast<const uint4*>(tp + va) + lane : nullptr;
+  uint4 cd[U], ct[U];
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        if (t0 + u < nt) {
-          if (HAS_D) cp_async16(slot_s + 512u * u, gd + go + 512 * u);
-          if (HAS_T) cp_async16(slot_s + 512u * (U + u), gt + go + 512 * u);
-        }
+  for (int u = 0; u < U; ++u) {
+    if (u < nt) {
+      if (HAS_D) cd[u] = ld_stream(gd + 32 * u);
+      if (HAS_T) ct[u] = ld_stream(gt + 32 * u);
+    }
+  }
+  for (int s = 0; s < nst; ++s) {
+    uint4 nd[U], nx[U];
+    const int t1 = (s + 1) * U;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (t1 + u < nt) {
+        if (HAS_D) nd[u] = ld_stream(gd + 32 * (t1 + u));
+        if (HAS_T) nx[u] = ld_stream(gt + 32 * (t1 + u));
       }
     }
-    cp_async_commit();
-  };
-#pragma unroll
-  for (int s = 0; s < kStagesRing; ++s) issue(s, ring_s + (uint32_t)(s * SLOT));
-  int slot = 0;
-  for (int s = 0; s < nst; ++s) {
-    cp_async_wait<kStagesRing - 1>();
-    const unsigned char* sl = lane_ring + slot * SLOT;
     const int t0 = s * U;
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       if (t0 + u < nt) {
         const int v = va + (lane + 32 * (t0 + u)) * VEC;
-        if (HAS_D) d_vec(ss.d, as_vec<T>(*reinterpret_cast<const uint4*>(sl + 512 * u)), v);
-        if (HAS_T) t_vec<SAMPLED>(ss.t, as_vec<T>(*reinterpret_cast<const uint4*>(sl + 512 * (U + u))), v, ss.c, beta);
+        if (HAS_D) d_vec(ss.d, as_vec<T>(cd[u]), v);
+        if (HAS_T) t_vec<SAMPLED>(ss.t, as_vec<T>(ct[u]), v, ss.c, beta);
       }
     }
-    issue(s + kStagesRing, ring_s + (uint32_t)(slot * SLOT));
-    slot = slot + 1 == kStagesRing ? 0 : slot + 1;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (HAS_D) cd[u] = nd[u];
+      if (HAS_T) ct[u] = nx[u];
+    }
   }
-  cp_async_wait<0>();
 }
 
 // ---- a warp's slice, segment by segment ------------------------------------------
 template <typename T, int MODE, bool SAMPLED>
 __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_begin, int64_t e_end,
-                           int64_t N, int Weff, int w, int lane, unsigned char* lane_ring) {
+                           int64_t N, int Weff, int w, int lane) {
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   const int beta = a.beta_rank > 0 ? a.beta_rank : 0;
@@ -842,7 +851,7 @@ __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_beg
       if (HAS_D) d_scalar(ss.d, Elem<T>::load(dp + v), v);
       if (HAS_T) t_scalar<SAMPLED>(ss.t, Elem<T>::load(tp + v), v, ss.c, beta);
     }
-    walk_body<T, MODE, SAMPLED>(ss, dp, tp, sg.va, sg.vb, beta, lane_ring, lane);
+    walk_body<T, MODE, SAMPLED>(ss, dp, tp, sg.va, sg.vb, beta, lane);
     if (lane < sg.v1 - sg.vb) {
       const int v = sg.vb + lane;
       if (HAS_D) d_scalar(ss.d, Elem<T>::load(dp + v), v);
@@ -867,8 +876,6 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
   const Workspace& W = a.ws;
   const bool ragged = a.k_row != nullptr;
   int* s_pref = reinterpret_cast<int*>(smem);
-  unsigned char* my_ring = smem + stream_pref_bytes(a.B, ragged) + (size_t)warp * kStagesRing * kStageWarpBytes +
-                          16 * lane;
 
   // -- present rows: exclusive prefix of k_row (ragged windows) -------------
   int nrows;
@@ -927,7 +934,7 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
   if (w >= Weff) return;
   const int64_t e_begin = split_start(w, N, Weff, VEC);
   const int64_t e_end = split_start(w + 1, N, Weff, VEC);
-  walk_slice<T, MODE, SAMPLED>(a, s_pref, e_begin, e_end, N, Weff, w, lane, my_ring);
+  walk_slice<T, MODE, SAMPLED>(a, s_pref, e_begin, e_end, N, Weff, w, lane);
 }
 
 // ---------------------------------------------------------------------------
@@ -1035,14 +1042,7 @@ __device__ __forceinline__ uint4 neg_inf_vec() {
                         : make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
 }
 
-// Entry k of a 16-byte vector (k may be a run-time value: selects, no local array).
-template <typename T>
-__device__ __forceinline__ float logit_at(uint4 q, int k) {
-  const int j = sizeof(T) == 2 ? (k >> 1) : k;
-  const uint32_t w = j == 0 ? q.x : j == 1 ? q.y : j == 2 ? q.z : q.w;
-  if (sizeof(T) == 2) return (k & 1) ? bf_hi(w) : bf_lo(w);
-  return __uint_as_float(w);
-}
+
 
 // Level 2 on group gm, whose logits sit in lanes own .. own+LPG-1 (vector
 // `sub` of the group in lane own+sub): every lane takes one entry, gathers its
