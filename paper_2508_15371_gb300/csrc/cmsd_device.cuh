@@ -83,7 +83,17 @@ __device__ __forceinline__ u64 mul2(u64 a, u64 b) {
 __device__ __forceinline__ u64 dup2(float x) { return pack2(x, x); }
 __device__ __forceinline__ u64 ex2_2(u64 x) { return pack2(ex2(lo32f(x)), ex2(hi32f(x))); }
 
-// ---- global loads -----------------------------------------------------------
+// ---- global memory ------------------------------------------------------------
+// GPU-scope add with acquire-release semantics: the caller's earlier stores
+// are visible before the add, and what other threads released before their
+// adds is visible after it.
+__device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
+  int old;
+  asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
+
 __device__ __forceinline__ uint4 ld_stream(const void* p) {
   uint4 r;
   asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"

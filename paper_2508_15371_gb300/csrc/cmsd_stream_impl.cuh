@@ -117,7 +117,8 @@ __device__ __forceinline__ void tlane_init(TLane& t, float c, int beta) {
   t.pos = kIntMax;
   t.posw = 0;
   t.cnt = 0;
-  t.thr = beta > 0 ? c : pos_inf();
+  t.thr = pos_inf();
+  if (beta > 0) t.thr = c;   // c is a pending load: read it only when needed
 }
 
 // move the exponent reference up to mx: s *= e^(ref - mx), t likewise
@@ -480,15 +481,6 @@ __device__ __forceinline__ void map_row(const StreamArgs& a, const int* pref, in
   i = ar - pref[lo];
 }
 
-__device__ __forceinline__ int checked_token(const StreamArgs& a, int r) {
-  int tok = __ldg(a.tokens + r);
-  if (tok < 0 || tok >= a.V) {
-    atomicOr(a.ws.err, 1u);
-    tok = 0;
-  }
-  return tok;
-}
-
 // Geometry of one segment: row elements [v0, v1), with the 16-byte aligned
 // body [va, vb) (a whole number of vectors) between a head and a tail.
 struct Seg {
@@ -591,7 +583,7 @@ __device__ void seq_epilogue(const StreamArgs& a, int b, int kb, int lane) {
 
 template <typename T, int MODE, bool SAMPLED>
 __device__ void row_results(const StreamArgs& a, int r, int b, int i, const DRed& d, const TRed& t,
-                            float c_tgt) {
+                            float c_tgt, float zd) {
   const Workspace& W = a.ws;
   float C = 0.f, MLd = 0.f, Sd = 1.f;
   if (MODE != kModeVerify) {
@@ -625,8 +617,6 @@ __device__ void row_results(const StreamArgs& a, int r, int b, int i, const DRed
       const float gap = t.m - c_tgt;
       acc = rank_ok && gap <= tau;
     } else {
-      const int tok = checked_token(a, r);
-      const float zd = Elem<T>::load((const T*)a.draft + (size_t)r * a.V + tok);
       const float p = exp2f(fmaf(c_tgt, kLog2e, -MLt)) / t.s;
       float q;
       if (MODE == kModeFused) {
@@ -680,13 +670,15 @@ struct SegState {
   DLane d;
   TLane t;
   float c;          // target logit at the drafted token
+  float zd;         // drafter logit at the drafted token (SAMPLED rule)
 };
 
 template <typename T, int MODE, bool SAMPLED>
-__device__ __forceinline__ void seg_begin(SegState<T>& ss, float c_tgt, int beta) {
+__device__ __forceinline__ void seg_begin(SegState<T>& ss, float c_tgt, float zd, int beta) {
   dlane_init(ss.d);
   tlane_init(ss.t, c_tgt, beta);
   ss.c = c_tgt;
+  ss.zd = zd;
 }
 
 // End of a segment (row ar / storage row r / sequence b, position i, len
@@ -725,20 +717,22 @@ __device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, 
     const int idx = (t.M == M && t.posw) ? first_equal<T>(tp, t.pos, t.posw, t.M, false) : kIntMax;
     tr = reduce_t(TRed{t.M, SAMPLED ? t_final(t) : 0.f, idx, t.cnt});
   }
+  // lane 0 stores the partial and counts it with a release; the warp that
+  // completes the row sees every other slice's partial through the acquire
+  // of its own count (extended to the other lanes by __syncwarp)
+  int old = 0;
   if (lane == 0) {
     Partial p;
     p.d_m = dr.m; p.d_s = dr.s; p.d_t2 = dr.t2; p.d_top2 = dr.top2; p.d_idx = dr.idx;
     p.t_m = tr.m; p.t_s = tr.s; p.t_idx = tr.idx; p.t_cnt = tr.cnt;
     p.pad[0] = p.pad[1] = p.pad[2] = 0;
     W.part[ar + w] = p;
+    old = atom_add_acq_rel(W.row_done + r, len);
   }
-  __threadfence();
-  int old = 0;
-  if (lane == 0) old = atomicAdd(W.row_done + r, len);
   old = __shfl_sync(kFull, old, 0);
   if (old + len != a.V) return;
   // -- this warp completed row r: merge every slice's partial -----------------
-  __threadfence();
+  __syncwarp();
   const int wf = find_warp((int64_t)ar * a.V, N, Weff, VEC);
   const int wl = find_warp((int64_t)ar * a.V + a.V - 1, N, Weff, VEC);
   DRed dm = dred_empty();
@@ -751,24 +745,18 @@ __device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, 
   }
   if (HAS_D) dr = reduce_d(dm);
   if (HAS_T) tr = reduce_t(tm);
-  if (lane == 0) {
-    W.row_done[r] = 0;
-    row_results<T, MODE, SAMPLED>(a, r, b, i, dr, tr, ss.c);
-  }
-  __threadfence();
   const int kb = k_of(a, b);
   int sold = 0;
-  if (lane == 0) sold = atomicAdd(W.seq_done + b, 1);
+  if (lane == 0) {
+    W.row_done[r] = 0;
+    row_results<T, MODE, SAMPLED>(a, r, b, i, dr, tr, ss.c, ss.zd);
+    sold = atom_add_acq_rel(W.seq_done + b, 1);
+  }
   sold = __shfl_sync(kFull, sold, 0);
   if (sold + 1 == kb) {
-    __threadfence();
+    __syncwarp();
     seq_epilogue<MODE, SAMPLED>(a, b, kb, lane);
   }
-}
-
-template <typename T>
-__device__ __forceinline__ float target_at_token(const StreamArgs& a, int r) {
-  return Elem<T>::load((const T*)a.target + (size_t)r * (size_t)a.V + checked_token(a, r));
 }
 
 // ---- one segment body, pipelined ----------------------------------------------
@@ -778,55 +766,72 @@ __device__ __forceinline__ float target_at_token(const StreamArgs& a, int r) {
 #ifndef CMSD_UNROLL
 #define CMSD_UNROLL 2
 #endif
-template <typename T, int MODE, bool SAMPLED>
-__device__ __forceinline__ void walk_body(SegState<T>& ss, const T* dp, const T* tp, int va, int vb, int beta,
-                                          int lane) {
+template <typename T>
+struct Pipe {
+  uint4 d[CMSD_UNROLL], t[CMSD_UNROLL];   // the stage in flight
+  const uint4* gd;
+  const uint4* gt;
+  int nt, nst;                            // this lane's vectors; warp-uniform stages
+};
+
+// issue the loads of stage 0
+template <typename T, int MODE>
+__device__ __forceinline__ void pipe_start(Pipe<T>& p, const T* dp, const T* tp, int va, int vb, int lane) {
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   constexpr int VEC = Elem<T>::kVec;
   constexpr int U = CMSD_UNROLL;
   const int nvec = (vb - va) / VEC;
-  if (nvec <= 0) return;
-  const int nt = nvec > lane ? (nvec - lane + 31) / 32 : 0;
-  const int nst = (nvec + 32 * U - 1) / (32 * U);
-  const uint4* gd = reinterpret_cast<const uint4*>(dp + va) + lane;
-  const uint4* gt = HAS_T ? reinterpret_cast<const uint4*>(tp + va) + lane : nullptr;
-  uint4 cd[U], ct[U];
+  p.nt = nvec > lane ? (nvec - lane + 31) / 32 : 0;
+  p.nst = (nvec + 32 * U - 1) / (32 * U);
+  p.gd = reinterpret_cast<const uint4*>(dp + va) + lane;
+  p.gt = HAS_T ? reinterpret_cast<const uint4*>(tp + va) + lane : nullptr;
 #pragma unroll
   for (int u = 0; u < U; ++u) {
-    if (u < nt) {
-      if (HAS_D) cd[u] = ld_stream(gd + 32 * u);
-      if (HAS_T) ct[u] = ld_stream(gt + 32 * u);
+    if (u < p.nt) {
+      if (HAS_D) p.d[u] = ld_stream(p.gd + 32 * u);
+      if (HAS_T) p.t[u] = ld_stream(p.gt + 32 * u);
     }
   }
-  for (int s = 0; s < nst; ++s) {
+}
+
+template <typename T, int MODE, bool SAMPLED>
+__device__ __forceinline__ void pipe_run(Pipe<T>& p, SegState<T>& ss, int va, int beta, int lane) {
+  constexpr bool HAS_D = MODE != kModeVerify;
+  constexpr bool HAS_T = MODE != kModeConf;
+  constexpr int VEC = Elem<T>::kVec;
+  constexpr int U = CMSD_UNROLL;
+  for (int s = 0; s < p.nst; ++s) {
     uint4 nd[U], nx[U];
     const int t1 = (s + 1) * U;
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      if (t1 + u < nt) {
-        if (HAS_D) nd[u] = ld_stream(gd + 32 * (t1 + u));
-        if (HAS_T) nx[u] = ld_stream(gt + 32 * (t1 + u));
+      if (t1 + u < p.nt) {
+        if (HAS_D) nd[u] = ld_stream(p.gd + 32 * (t1 + u));
+        if (HAS_T) nx[u] = ld_stream(p.gt + 32 * (t1 + u));
       }
     }
     const int t0 = s * U;
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      if (t0 + u < nt) {
+      if (t0 + u < p.nt) {
         const int v = va + (lane + 32 * (t0 + u)) * VEC;
-        if (HAS_D) d_vec(ss.d, as_vec<T>(cd[u]), v);
-        if (HAS_T) t_vec<SAMPLED>(ss.t, as_vec<T>(ct[u]), v, ss.c, beta);
+        if (HAS_D) d_vec(ss.d, as_vec<T>(p.d[u]), v);
+        if (HAS_T) t_vec<SAMPLED>(ss.t, as_vec<T>(p.t[u]), v, ss.c, beta);
       }
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      if (HAS_D) cd[u] = nd[u];
-      if (HAS_T) ct[u] = nx[u];
+      if (HAS_D) p.d[u] = nd[u];
+      if (HAS_T) p.t[u] = nx[u];
     }
   }
 }
 
 // ---- a warp's slice, segment by segment ------------------------------------------
+// Order of a segment's start: its first stage of logits is requested, then
+// the logits at its drafted token (whose index was requested one segment
+// earlier), so the slice's first loads are not held up behind the token.
 template <typename T, int MODE, bool SAMPLED>
 __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_begin, int64_t e_end,
                            int64_t N, int Weff, int w, int lane) {
@@ -834,8 +839,8 @@ __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_beg
   constexpr bool HAS_T = MODE != kModeConf;
   const int beta = a.beta_rank > 0 ? a.beta_rank : 0;
   const void* base = HAS_D ? a.draft : a.target;
-  float c_next = 0.f;
-  if (HAS_T) c_next = target_at_token<T>(a, make_seg<T>(a, s_pref, e_begin, e_end, base).r);
+  int tok_next = 0;
+  if (HAS_T) tok_next = __ldg(a.tokens + make_seg<T>(a, s_pref, e_begin, e_end, base).r);
   for (int64_t e0 = e_begin; e0 < e_end;) {
     const Seg sg = make_seg<T>(a, s_pref, e0, e_end, base);
     const int len = sg.v1 - sg.v0;
@@ -843,15 +848,27 @@ __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_beg
     const size_t rowoff = (size_t)sg.r * (size_t)a.V;
     const T* dp = (const T*)a.draft + rowoff;
     const T* tp = HAS_T ? (const T*)a.target + rowoff : nullptr;
+    Pipe<T> pp;
+    pipe_start<T, MODE>(pp, dp, tp, sg.va, sg.vb, lane);
+    float c = 0.f, zd = 0.f;
+    if (HAS_T) {
+      int tok = tok_next;
+      if (e0 < e_end) tok_next = __ldg(a.tokens + make_seg<T>(a, s_pref, e0, e_end, base).r);
+      if (tok < 0 || tok >= a.V) {
+        if (lane == 0) atomicOr(a.ws.err, 1u);
+        tok = 0;
+      }
+      c = Elem<T>::load(tp + tok);
+      if (SAMPLED) zd = Elem<T>::load(dp + tok);
+    }
     SegState<T> ss;
-    seg_begin<T, MODE, SAMPLED>(ss, c_next, beta);
-    if (HAS_T && e0 < e_end) c_next = target_at_token<T>(a, make_seg<T>(a, s_pref, e0, e_end, base).r);
+    seg_begin<T, MODE, SAMPLED>(ss, c, zd, beta);
     if (lane < sg.va - sg.v0) {
       const int v = sg.v0 + lane;
       if (HAS_D) d_scalar(ss.d, Elem<T>::load(dp + v), v);
       if (HAS_T) t_scalar<SAMPLED>(ss.t, Elem<T>::load(tp + v), v, ss.c, beta);
     }
-    walk_body<T, MODE, SAMPLED>(ss, dp, tp, sg.va, sg.vb, beta, lane);
+    pipe_run<T, MODE, SAMPLED>(pp, ss, sg.va, beta, lane);
     if (lane < sg.v1 - sg.vb) {
       const int v = sg.vb + lane;
       if (HAS_D) d_scalar(ss.d, Elem<T>::load(dp + v), v);
@@ -1003,14 +1020,6 @@ __device__ __forceinline__ float resid_vec(uint4 qt, uint4 qd, const RowStat& s)
   return lo32f(acc) + hi32f(acc);
 }
 
-// GPU-scope add with acquire-release semantics: the caller's earlier stores
-// are visible before the add, and what other threads released before their
-// adds is visible after it.
-__device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
-  int old;
-  asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
-  return old;
-}
 
 // 16 bytes of logits at entry v of one row: one vector load when the vector is
 // aligned and inside the row, else element loads with entries past the row
