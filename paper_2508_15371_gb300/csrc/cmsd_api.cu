@@ -220,7 +220,7 @@ int launch(int dtype, int mode, bool sampled, StreamArgs& a, void* ws, size_t ws
   int grid = 0;
   rc = stream_grid(dtype, mode, sampled, smem, &grid);
   if (rc) return rc;
-  a.nwarps = grid * kWarpsPerBlock;
+  a.nwarps = grid * kStreamWarps;
   prof_record(0, s);
   cudaError_t e = dtype == CMSD_F32 ? launch_stream_f32(mode, sampled, a, grid, smem, s)
                                     : launch_stream_bf16(mode, sampled, a, grid, smem, s);
@@ -426,7 +426,7 @@ int cmsd_launch_info(int dtype, int* warps_out, int* sms_out) {
   if (rc) return rc;
   rc = stream_grid(dtype, kModeFused, true, stream_smem_bytes(0, false), &grid);
   if (rc) return rc;
-  if (warps_out) *warps_out = grid * kWarpsPerBlock;
+  if (warps_out) *warps_out = grid * kStreamWarps;
   if (sms_out) *sms_out = sms;
   return CMSD_OK;
 }

@@ -5,8 +5,15 @@
 
 namespace cmsd {
 
-constexpr int kThreads = 256;                 // threads per CTA
+constexpr int kThreads = 256;                 // threads per CTA (resample kernel)
 constexpr int kWarpsPerBlock = kThreads / 32;
+// The streaming kernel runs as few, large CTAs (one per SM by default): warps
+// of one CTA are scheduled evenly, warps of co-resident CTAs are not.
+#ifndef CMSD_STREAM_THREADS
+#define CMSD_STREAM_THREADS 768
+#endif
+constexpr int kStreamThreads = CMSD_STREAM_THREADS;
+constexpr int kStreamWarps = kStreamThreads / 32;
 constexpr int kMaxWarpsPerSM = 64;            // 2048 threads / SM
 constexpr int kMaxRaggedB = 12000;            // B limit when k_row is given (prefix in smem)
 

@@ -422,22 +422,6 @@ __device__ __forceinline__ int64_t stream_min_len(int V) {
   const int64_t a = (int64_t)V / 64 + 64;
   return a > 2048 ? a : 2048;
 }
-__device__ __forceinline__ int64_t stream_cta_min_len(int V) {
-  const int64_t a = (int64_t)V / 16 + 64;
-  return a > 16384 ? a : 16384;
-}
-__device__ __forceinline__ int64_t split_start(int w, int64_t N, int W, int vec) {
-  if (w >= W) return N;
-  return ((int64_t)w * N / W) & ~(int64_t)(vec - 1);
-}
-__device__ __forceinline__ int find_warp(int64_t e, int64_t N, int W, int vec) {
-  int w = (int)((e * (int64_t)W) / N);
-  if (w >= W) w = W - 1;
-  while (w + 1 < W && split_start(w + 1, N, W, vec) <= e) ++w;
-  while (w > 0 && split_start(w, N, W, vec) > e) --w;
-  return w;
-}
-
 // a / b for 0 <= a, 0 < b, in 32-bit arithmetic when both fit.
 __device__ __forceinline__ int64_t div_nn(int64_t a, int64_t b) {
   if (a <= 0x7FFFFFFF && b <= 0x7FFFFFFF) return (int64_t)((uint32_t)a / (uint32_t)b);
@@ -456,6 +440,69 @@ struct EvenSplit {
   __device__ int owner(int64_t u) const {
     const int64_t big = (q + 1) * rem;
     return u < big ? (int)div_nn(u, q + 1) : rem + (int)div_nn(u - big, q);
+  }
+};
+
+// How the present-row stream (R rows of V logits, N = R*V elements) is cut
+// into warp slices.  When there are at least as many warps as rows, each row
+// is cut into wpr pieces of one warp each (no slice crosses a row end, so
+// every warp streams one segment); otherwise the stream is cut into W equal
+// runs of 16-byte vectors.  Slices start on multiples of VEC elements (the
+// last one ends at N).
+struct StreamSplit {
+  int64_t N;
+  int W;          // warps with work
+  int V, VEC;
+  int wpr;        // > 0: row-aligned split with wpr warps per row
+  int qv, rv;     // row-aligned: V / wpr, V % wpr
+  int64_t q;      // flat: vectors per warp (the first rem warps one more)
+  int rem;
+  __device__ StreamSplit(int R, int V_, int vec, int nwarps, int64_t min_len) {
+    V = V_;
+    VEC = vec;
+    N = (int64_t)R * V;
+    int64_t want = N / min_len;
+    if (want < 1) want = 1;
+    const int Wmax = (int)(want < nwarps ? want : nwarps);
+    int p = nwarps / R;                              // pieces per row that fit
+    const int64_t pm = (int64_t)V / min_len;
+    const int pmax = pm > 0 ? (int)pm : 1;
+    if (p > pmax) p = pmax;
+    if (p >= 1 && (int64_t)p * R * 8 >= (int64_t)Wmax * 7) {   // uses at least 7/8 of the warps
+      wpr = p;
+      W = p * R;
+      qv = V / p;
+      rv = V - qv * p;
+      q = 0;
+      rem = 0;
+    } else {
+      wpr = 0;
+      W = Wmax;
+      qv = rv = 0;
+      const int64_t nv = N / VEC;
+      q = div_nn(nv, W);
+      rem = (int)(nv - q * W);
+    }
+  }
+  __device__ int64_t start(int w) const {
+    if (w >= W) return N;
+    if (wpr > 0) {
+      const int row = w / wpr, k = w - row * wpr;
+      const int off = k * qv + (k < rv ? k : rv);
+      return (int64_t)row * V + (off & ~(VEC - 1));
+    }
+    return ((int64_t)w * q + (w < rem ? w : rem)) * VEC;
+  }
+  // warps holding the first and the last element of row ar
+  __device__ int first_warp(int ar) const { return wpr > 0 ? ar * wpr : owner_flat((int64_t)ar * V); }
+  __device__ int last_warp(int ar) const {
+    return wpr > 0 ? ar * wpr + wpr - 1 : owner_flat((int64_t)ar * V + V - 1);
+  }
+  __device__ int owner_flat(int64_t e) const {
+    const int64_t ev = e / VEC;
+    const int64_t big = (q + 1) * rem;
+    const int w = ev < big ? (int)div_nn(ev, q + 1) : rem + (int)div_nn(ev - big, q);
+    return w < W ? w : W - 1;
   }
 };
 
@@ -661,7 +708,7 @@ template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 #ifndef CMSD_MIN_BLOCKS
-#define CMSD_MIN_BLOCKS 3
+#define CMSD_MIN_BLOCKS 1
 #endif
 
 // Running state of the segment a warp is reducing.
@@ -686,7 +733,7 @@ __device__ __forceinline__ void seg_begin(SegState<T>& ss, float c_tgt, float zd
 // sequence epilogue if this warp completes them.
 template <typename T, int MODE, bool SAMPLED>
 __device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, int b, int i, int len,
-                           int64_t N, int Weff, int w, int lane) {
+                           const StreamSplit& sp, int w, int lane) {
   const T* dp = (const T*)a.draft + (size_t)r * (size_t)a.V;
   const T* tp = (MODE != kModeConf) ? (const T*)a.target + (size_t)r * (size_t)a.V : nullptr;
   constexpr bool HAS_D = MODE != kModeVerify;
@@ -733,8 +780,8 @@ __device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, 
   if (old + len != a.V) return;
   // -- this warp completed row r: merge every slice's partial -----------------
   __syncwarp();
-  const int wf = find_warp((int64_t)ar * a.V, N, Weff, VEC);
-  const int wl = find_warp((int64_t)ar * a.V + a.V - 1, N, Weff, VEC);
+  const int wf = sp.first_warp(ar);
+  const int wl = sp.last_warp(ar);
   DRed dm = dred_empty();
   TRed tm = tred_empty();
   for (int k = wf + lane; k <= wl; k += 32) {
@@ -834,7 +881,7 @@ __device__ __forceinline__ void pipe_run(Pipe<T>& p, SegState<T>& ss, int va, in
 // earlier), so the slice's first loads are not held up behind the token.
 template <typename T, int MODE, bool SAMPLED>
 __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_begin, int64_t e_end,
-                           int64_t N, int Weff, int w, int lane) {
+                           const StreamSplit& sp, int w, int lane) {
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   const int beta = a.beta_rank > 0 ? a.beta_rank : 0;
@@ -874,12 +921,12 @@ __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_beg
       if (HAS_D) d_scalar(ss.d, Elem<T>::load(dp + v), v);
       if (HAS_T) t_scalar<SAMPLED>(ss.t, Elem<T>::load(tp + v), v, ss.c, beta);
     }
-    seg_finish<T, MODE, SAMPLED>(a, ss, sg.ar, sg.r, sg.b, sg.i, len, N, Weff, w, lane);
+    seg_finish<T, MODE, SAMPLED>(a, ss, sg.ar, sg.r, sg.b, sg.i, len, sp, w, lane);
   }
 }
 
 template <typename T, int MODE, bool SAMPLED>
-__global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const StreamArgs a) {
+__global__ void __launch_bounds__(kStreamThreads, CMSD_MIN_BLOCKS) stream_kernel(const StreamArgs a) {
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   constexpr int VEC = Elem<T>::kVec;
@@ -897,7 +944,7 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
   // -- present rows: exclusive prefix of k_row (ragged windows) -------------
   int nrows;
   if (ragged) {
-    const int per = (a.B + kThreads - 1) / kThreads;
+    const int per = (a.B + kStreamThreads - 1) / kStreamThreads;
     const int b0 = threadIdx.x * per;
     int tot = 0;
     for (int b = b0; b < b0 + per && b < a.B; ++b) tot += k_of(a, b);
@@ -907,7 +954,7 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
       const int y = __shfl_up_sync(kFull, incl, o);
       if (lane >= o) incl += y;
     }
-    __shared__ int s_wsum[kWarpsPerBlock];
+    __shared__ int s_wsum[kStreamWarps];
     if (lane == 31) s_wsum[warp] = incl;
     __syncthreads();
     int wofs = 0;
@@ -917,7 +964,7 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
       s_pref[b] = run;
       run += k_of(a, b);
     }
-    if (threadIdx.x == kThreads - 1) s_pref[a.B] = run;
+    if (threadIdx.x == kStreamThreads - 1) s_pref[a.B] = run;
     __syncthreads();
     nrows = s_pref[a.B];
   } else {
@@ -926,8 +973,8 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
 
   // -- sequences with no present position, and k_row range errors -----------
   if (ragged) {
-    const int gt = blockIdx.x * kThreads + threadIdx.x;
-    const int gn = gridDim.x * kThreads;
+    const int gt = blockIdx.x * kStreamThreads + threadIdx.x;
+    const int gn = gridDim.x * kStreamThreads;
     for (int b = gt; b < a.B; b += gn) {
       const int raw = __ldg(a.k_row + b);
       if (raw < 0 || raw > a.K) atomicOr(W.err, 2u);
@@ -944,14 +991,14 @@ __global__ void __launch_bounds__(kThreads, CMSD_MIN_BLOCKS) stream_kernel(const
     }
   }
 
-  const int64_t N = (int64_t)nrows * a.V;
-  if (N == 0) return;
-  const int Weff = eff_warps(N, stream_min_len(a.V), a.nwarps);
-  const int w = blockIdx.x * kWarpsPerBlock + warp;
-  if (w >= Weff) return;
-  const int64_t e_begin = split_start(w, N, Weff, VEC);
-  const int64_t e_end = split_start(w + 1, N, Weff, VEC);
-  walk_slice<T, MODE, SAMPLED>(a, s_pref, e_begin, e_end, N, Weff, w, lane);
+  if (nrows == 0) return;
+  const StreamSplit sp(nrows, a.V, VEC, a.nwarps, stream_min_len(a.V));
+  const int w = blockIdx.x * kStreamWarps + warp;
+  if (w >= sp.W) return;
+  const int64_t e_begin = sp.start(w);
+  const int64_t e_end = sp.start(w + 1);
+  if (e_begin >= e_end) return;
+  walk_slice<T, MODE, SAMPLED>(a, s_pref, e_begin, e_end, sp, w, lane);
 }
 
 // ---------------------------------------------------------------------------
@@ -1280,7 +1327,7 @@ cudaError_t launch_stream_t(int mode, bool sampled, const StreamArgs& a, int gri
   do {                                                                                        \
     cudaFuncSetAttribute(stream_kernel<T, M, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
                          (int)smem);                                                          \
-    stream_kernel<T, M, S><<<grid, kThreads, smem, s>>>(a);                                   \
+    stream_kernel<T, M, S><<<grid, kStreamThreads, smem, s>>>(a);                                   \
   } while (0)
   if (mode == kModeConf) CMSD_L(kModeConf, false);
   else if (mode == kModeVerify) { if (sampled) CMSD_L(kModeVerify, true); else CMSD_L(kModeVerify, false); }
@@ -1294,7 +1341,7 @@ cudaError_t occupancy_stream_t(int mode, bool sampled, size_t smem, int* nb) {
 #define CMSD_O(M, S)                                                                            \
   (cudaFuncSetAttribute(stream_kernel<T, M, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,   \
                         (int)smem),                                                            \
-   cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, stream_kernel<T, M, S>, kThreads, smem))
+   cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, stream_kernel<T, M, S>, kStreamThreads, smem))
   if (mode == kModeConf) return CMSD_O(kModeConf, false);
   if (mode == kModeVerify) return sampled ? CMSD_O(kModeVerify, true) : CMSD_O(kModeVerify, false);
   return sampled ? CMSD_O(kModeFused, true) : CMSD_O(kModeFused, false);
