@@ -5,7 +5,10 @@
 
 namespace cmsd {
 
-constexpr int kThreads = 256;                 // threads per CTA (resample kernel)
+#ifndef CMSD_RES_THREADS
+#define CMSD_RES_THREADS 256
+#endif
+constexpr int kThreads = CMSD_RES_THREADS;    // threads per CTA (resample kernel)
 constexpr int kWarpsPerBlock = kThreads / 32;
 // The streaming kernel runs as few, large CTAs (one per SM by default): warps
 // of one CTA are scheduled evenly, warps of co-resident CTAs are not.

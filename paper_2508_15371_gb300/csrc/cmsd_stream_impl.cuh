@@ -301,18 +301,21 @@ __device__ __forceinline__ float logit_at(uint4 q, int k) {
 // is one aligned 16-byte vector of the row: it is read with a single load
 // and searched in registers.
 template <typename T>
-__device__ __forceinline__ int first_equal(const T* row, int pos, int w, float m, bool clamp) {
-  if (w <= 1) return pos;
-  const uint4 q = __ldcg(reinterpret_cast<const uint4*>(row + pos));
+__device__ __forceinline__ int first_in_vec(uint4 q, float m, bool clamp) {
   const float nc = neg_clamp();
-  int k = w;
+  int k = 0;
 #pragma unroll
   for (int j = Elem<T>::kVec - 1; j >= 0; --j) {
     float z = logit_at<T>(q, j);
     if (clamp) z = fmaxf(z, nc);
     k = (z == m) ? j : k;
   }
-  return k < w ? pos + k : pos;
+  return k;
+}
+template <typename T>
+__device__ __forceinline__ int first_equal(const T* row, int pos, int w, float m, bool clamp) {
+  if (w <= 1) return pos;
+  return pos + first_in_vec<T>(__ldcg(reinterpret_cast<const uint4*>(row + pos)), m, clamp);
 }
 
 // ---------------------------------------------------------------------------
@@ -562,6 +565,66 @@ template <int MODE, bool SAMPLED>
 __device__ void seq_epilogue(const StreamArgs& a, int b, int kb, int lane) {
   const Workspace& W = a.ws;
   const int base = b * a.K;
+  if (a.K <= 32) {
+    // one position per lane: every value the outputs need is requested at once
+    const int i = lane;
+    const bool valid = i < kb;
+    int acc = 1, tok = -1, tmx = 0;
+    float cf = 0.f;
+    float2 ts = make_float2(0.f, 1.f), ds = make_float2(0.f, 1.f);
+    if (valid) {
+      if (MODE != kModeConf) {
+        acc = __ldcg(W.row_acc + base + i);
+        tok = __ldg(a.tokens + base + i);
+        tmx = __ldcg(W.row_targmax + base + i);
+        if (SAMPLED) {
+          ts = __ldcg(W.row_tstat + base + i);
+          ds = __ldcg(W.row_dstat + base + i);
+        }
+      }
+      if (MODE != kModeVerify) cf = __ldcg(W.row_conf + base + i);
+    }
+    const unsigned rej = __ballot_sync(kFull, valid && !acc);
+    const int n = rej ? __ffs(rej) - 1 : kb;
+    if (MODE != kModeVerify) {
+      const float csum = warp_sum_f(cf);
+      if (lane == 0 && a.k_next) {
+        int k = a.k_min;
+        if (kb > 0) {
+          const float cbar = csum / (float)kb;
+          const float x = a.alpha * cbar * (float)a.k_max;
+          k = (int)floorf(x);
+          k = k < a.k_min ? a.k_min : (k > a.k_max ? a.k_max : k);
+        }
+        a.k_next[b] = k;
+      }
+    }
+    if (MODE != kModeConf) {
+      if (i < a.K) {
+        int ot = -1;
+        if (i < n) ot = tok;
+        else if (i == n && n < kb) ot = SAMPLED ? -1 : tmx;
+        a.out_tokens[base + i] = ot;
+        if (a.accept) a.accept[base + i] = valid ? (unsigned char)(acc != 0) : 0;
+      }
+      if (lane == 0) a.n_accept[b] = n;
+      if (SAMPLED && i == n && n < kb) {
+        const int slot = atomicAdd(W.rej_count, 1);
+        if (slot < a.B) {
+          RejRec q;
+          q.r = base + n; q.b = b; q.n = n;
+          q.targmax = tmx;
+          q.MLt = ts.x; q.invSt = 1.0f / ts.y;
+          q.MLd = ds.x; q.invSd = 1.0f / ds.y;
+          W.rej[slot] = q;
+        } else {
+          atomicOr(W.err, 4u);   // queue not drained by a previous call: workspace misuse
+        }
+      }
+    }
+    if (lane == 0) W.seq_done[b] = 0;
+    return;
+  }
   int n = kb;
   float csum = 0.f;
   for (int i0 = 0; i0 < kb; i0 += 32) {
@@ -623,6 +686,7 @@ __device__ void seq_epilogue(const StreamArgs& a, int b, int kb, int lane) {
   }
   if (lane == 0) W.seq_done[b] = 0;
 }
+
 
 // ---------------------------------------------------------------------------
 // row results from the merged statistics
@@ -738,7 +802,6 @@ __device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, 
   const T* tp = (MODE != kModeConf) ? (const T*)a.target + (size_t)r * (size_t)a.V : nullptr;
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
-  constexpr int VEC = Elem<T>::kVec;
   const Workspace& W = a.ws;
   DRed dr = dred_empty();
   TRed tr = tred_empty();

@@ -71,11 +71,11 @@ def test_static_scratch_matches_workspace_entry_point(cmsd, name, kw, rule, k_ro
 
 
 def test_static_scratch_rejects_oversize_problem(cmsd):
-    # B*K = 65536 positions needs more than CMSD_STATIC_SCRATCH_BYTES; the call
+    # B*K = 131072 positions needs more than CMSD_STATIC_SCRATCH_BYTES; the call
     # is refused on the host before any pointer is used or anything enqueued.
     p = cmsd.params(8, "sampled")
     rc = cmsd.lib().cmsd_confidence_verify_static(
-        None, None, None, None, 64, 1024, 32000, cmsd.BF16, ctypes.byref(p), 0, 0,
+        None, None, None, None, 128, 1024, 32000, cmsd.BF16, ctypes.byref(p), 0, 0,
         None, None, None, None, None, None, None, None, None, None)
     assert rc == cmsd.ESCRATCH
     assert b"static scratch" in cmsd.lib().cmsd_strerror(rc)
