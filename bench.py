@@ -356,6 +356,11 @@ def run_ours(args):
             dist.destroy_process_group()
         return 0
 
+    # ---- decode-loop simulation (rank 0, N = 1 only) -------------------------
+    dsim = None
+    if world == 1 and not args.no_decode_sim:
+        dsim = decode_sim_report()
+
     # ---- CPU oracle baseline (rank 0, N = 1 only) ---------------------------
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
@@ -388,10 +393,39 @@ def run_ours(args):
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk,
     }
+    if dsim is not None:
+        line["decode_sim"] = dsim
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
     return 0
+
+
+def decode_sim_report(B=32, K=16, V=32000, iterations=512):
+    """Algorithm 1 as a decode loop over device-generated f32 logits: k_next of
+    each iteration is the next iteration's k_row.  Timed with CUDA events over
+    all iterations (logit generation included)."""
+    import torch
+    from paper_2508_15371_gb300 import cmsd, decode_sim
+    p = cmsd.params(K, "sampled")
+    sim = decode_sim.DecodeSim(B, K, V, iterations, p, seed=4)
+    for it in range(3):
+        sim.step(it)
+    torch.cuda.synchronize()
+    sim = decode_sim.DecodeSim(B, K, V, iterations, p, seed=4)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for it in range(iterations):
+        sim.step(it)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    hist = {"k": sim.hist_k.cpu().numpy(), "n_accept": sim.hist_n.cpu().numpy()}
+    s = decode_sim.summarize(hist)
+    s.update({"workload": f"B={B} K_max={K} V={V} f32, {iterations} iterations, sampled rule, AR(1) spike heights",
+              "ms_per_iteration": ms / iterations, "rows_per_s": s["rows"] / (ms * 1e-3),
+              "timing": "CUDA events over the loop, device logit generation included"})
+    return s
 
 
 def main():
@@ -403,6 +437,7 @@ def main():
     ap.add_argument("--rule", choices=["sampled", "paper"], default="sampled")
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-decode-sim", action="store_true", help="skip the decode-loop simulation report")
     ap.add_argument("--load-window", type=float, default=0.8,
                     help="seconds of untimed steps just before the timed region (clock sampling)")
     args = ap.parse_args()
