@@ -10,6 +10,7 @@ from .cmsd_oracle import (  # noqa: F401
     accept_paper,
     accept_sampled,
     bf16_bits_to_f64,
+    bonus_token,
     confidence,
     confidence_verify,
     decode_sim_sequence,
@@ -21,6 +22,7 @@ from .cmsd_oracle import (  # noqa: F401
     residual_token,
     softmax,
     tau_t,
+    two_level_race,
     unified_confidence,
     verify,
     verify_sequence,

@@ -27,8 +27,8 @@ Steps and where the paper defines them:
                     residual max(0, p - q) with a two-level exponential race
                     (groups of 32 entries, then entries of the winning group).
 
-Readings where the paper is garbled, silent or self-contradictory (each is
-listed with its reason in the design doc):
+Readings where the paper is garbled, silent or self-contradictory (the
+reason for each is stated beside it):
   C1  the entropy term enters the ensemble as 1 - H/log|V| (high entropy is
       low confidence, Sec. III.B(b) "low entropy ... Cbar -> 1").
   C2  the garbled "sigma * (beta * (z1 - z2))" is the logistic
@@ -43,7 +43,14 @@ listed with its reason in the design doc):
       logits; z(2) is the largest logit at any index other than argmax.
   C9  SAMPLED acceptance probability min(1, e^tau p/q), residual
       max(0, p - q) (tau = 0 gives exact speculative sampling).
-  C10 no bonus token: when all k positions are accepted no token is added.
+  C10 bonus row (optional, Params.bonus): the verifier scores one position
+      more than was drafted (Sec. III.A(2): after the accepted prefix the
+      verifier's own prediction continues the sequence); when all k drafts
+      are accepted, that row gives one more token -- its argmax under the
+      PAPER rule, a draw from its softmax under the SAMPLED rule.  Without
+      it, no token is added when all k positions are accepted.
+  T3  fixed draft length (Params.k_fixed > 0): the "fixed k" variants of the
+      ablation in Sec. IV (Table III) replace the adaptive k by a constant.
   C12 uniforms from Philox4x32-10 (oracle/philox.py).
   C13 -inf logits have probability 0 and add nothing to the entropy.
   R1  when the residual is identically zero (possible only with the rank
@@ -82,6 +89,8 @@ class Params:
     gamma: float = 1.0
     tau_sign: int = 1           # +1: printed equation; -1: prose reading
     rule: str = "paper"         # "paper" or "sampled"
+    k_fixed: int = 0            # > 0: constant draft length (Table III "fixed k")
+    bonus: bool = False         # the verifier supplies row k_b after the drafts
 
 
 # ---------------------------------------------------------------------------
@@ -168,6 +177,8 @@ def next_draft_length(C_window, P: Params):
 
     Returns (k, flagged).  An empty window gives k_min (no signal).
     """
+    if P.k_fixed > 0:                          # Table III, fixed k: no adaptation
+        return int(P.k_fixed), False
     C_window = [float(c) for c in C_window]
     if not C_window:
         return P.k_min, False
@@ -248,28 +259,22 @@ def _race(keys_E, rates, eps=FLAG_EPS, r_lo=None, r_hi=None):
     return w, bool(key_hi_w >= np.min(key_lo))
 
 
-def residual_token(zt, zd, seed, b, n, iteration):
-    """Draw from norm(max(0, p - q)) with a two-level exponential race.
+def two_level_race(r, r_lo, r_hi, seed, b, n, iteration):
+    """Draw from norm(r) (r >= 0, not all 0) with a two-level exponential race.
 
-    r_v = max(0, p_v - q_v); the vocabulary is cut into groups of
-    philox.GROUP = 32 consecutive entries with mass R_g = sum of r_v over the
-    group.  Level 1: group g gets E_g = -log(1 - U_g) and the winning group is
-    argmin E_g / R_g (law R_g / R).  Level 2: inside the winning group, entry v
-    gets E_v = -log(1 - U_v) and the token is argmin E_v / r_v (law r_v / R_g).
-    Together the token has law r_v / R, the normalised residual.  Ties go to
-    the lowest index.  Returns (token, flagged); flagged when either level's
-    winner could change under relative perturbations of FLAG_EPS in p, q and
-    the exponentials.
+    The vocabulary is cut into groups of philox.GROUP = 32 consecutive
+    entries with mass R_g = sum of r_v over the group.  Level 1: group g gets
+    E_g = -log(1 - U_g) and the winning group is argmin E_g / R_g (law
+    R_g / R).  Level 2: inside the winning group, entry v gets
+    E_v = -log(1 - U_v) and the token is argmin E_v / r_v (law r_v / R_g).
+    Together the token has law r_v / R.  Ties go to the lowest index.  The
+    uniforms are those of position n of sequence b (oracle/philox.py).
+    Returns (token, flagged); flagged when either level's winner could change
+    with each rate anywhere in [r_lo, r_hi] and the exponentials perturbed by
+    a relative FLAG_EPS.
     """
-    p = softmax(zt)
-    q = softmax(zd)
-    V = p.size
-    r = np.maximum(0.0, p - q)
-    if not np.any(r > 0):
-        return int(np.argmax(np.asarray(zt, dtype=np.float64))), False   # reading R1
     eps = FLAG_EPS
-    r_hi = np.maximum(0.0, p * (1 + eps) - q * (1 - eps))
-    r_lo = np.maximum(0.0, p * (1 - eps) - q * (1 + eps))
+    V = r.size
     G = philox.GROUP
     ng = (V + G - 1) // G
     pad = ng * G - V
@@ -282,6 +287,40 @@ def residual_token(zt, zd, seed, b, n, iteration):
     Uv = philox.residual_uniforms(seed, b, n, iteration, V)[v0:v1]
     k, f2 = _race(-np.log1p(-Uv), r[v0:v1], eps, r_lo[v0:v1], r_hi[v0:v1])
     return v0 + k, bool(f1 or f2)
+
+
+def residual_token(zt, zd, seed, b, n, iteration):
+    """Draw from norm(max(0, p - q)) at the rejected position n (reading C9).
+
+    r_v = max(0, p_v - q_v) with p the verifier's and q the drafter's softmax;
+    the draw is the two-level race above.  If r is identically 0 the
+    correction is the verifier's argmax (reading R1).  Returns (token,
+    flagged); the rate bounds perturb p and q by a relative FLAG_EPS.
+    """
+    p = softmax(zt)
+    q = softmax(zd)
+    r = np.maximum(0.0, p - q)
+    if not np.any(r > 0):
+        return int(np.argmax(np.asarray(zt, dtype=np.float64))), False   # reading R1
+    eps = FLAG_EPS
+    r_hi = np.maximum(0.0, p * (1 + eps) - q * (1 - eps))
+    r_lo = np.maximum(0.0, p * (1 - eps) - q * (1 + eps))
+    return two_level_race(r, r_lo, r_hi, seed, b, n, iteration)
+
+
+def bonus_token(zt, rule, seed, b, n, iteration):
+    """The token of the verifier's extra row n = k_b when all drafts were
+    accepted (reading C10): its argmax (lowest index) under the PAPER rule,
+    a draw from its softmax p under the SAMPLED rule (the two-level race with
+    r = p, using the uniforms of position n, which no residual draw of this
+    iteration uses since a residual position is always below k_b).
+    Returns (token, flagged)."""
+    zt = np.asarray(zt, dtype=np.float64)
+    if rule == "paper":
+        return int(np.argmax(zt)), False
+    p = softmax(zt)
+    eps = FLAG_EPS
+    return two_level_race(p, p * (1 - eps), p * (1 + eps), seed, b, n, iteration)
 
 
 # ---------------------------------------------------------------------------
@@ -357,8 +396,10 @@ def confidence(draft, P: Params, k_row=None, rows=None):
 def verify_sequence(draft_b, target_b, tokens_b, conf_b, k_b, P: Params, seed, b, iteration):
     """Verification of one sequence: per-position accept, first failure, correction.
 
-    Returns dict with accept[k_b], acc_flag[k_b], n_accept, n_flag, out_tokens[K],
-    tok_flag, target_argmax[k_b].
+    With P.bonus the verifier rows target_b hold one more row than drafted
+    (row k_b is the bonus row, reading C10) and out_tokens has K + 1 entries.
+    Returns dict with accept[k_b], acc_flag[k_b], n_accept, n_flag,
+    out_tokens[K (+1)], tok_flag, target_argmax[k_b].
     """
     K = len(tokens_b)
     acc = np.zeros(k_b, dtype=bool)
@@ -383,7 +424,7 @@ def verify_sequence(draft_b, target_b, tokens_b, conf_b, k_b, P: Params, seed, b
             n = i
             break
     n_flag = bool(np.any(aflag[: min(n + 1, k_b)]))
-    out = np.full(K, -1, dtype=np.int64)
+    out = np.full(K + 1 if P.bonus else K, -1, dtype=np.int64)
     out[:n] = np.asarray(tokens_b[:n], dtype=np.int64)
     tok_flag = n_flag
     if n < k_b:
@@ -392,6 +433,9 @@ def verify_sequence(draft_b, target_b, tokens_b, conf_b, k_b, P: Params, seed, b
         else:
             out[n], rflag = residual_token(target_b[n], draft_b[n], seed, b, n, iteration)
             tok_flag = tok_flag or rflag
+    elif P.bonus:                               # every draft accepted: the verifier's own token
+        out[k_b], rflag = bonus_token(target_b[k_b], P.rule, seed, b, k_b, iteration)
+        tok_flag = tok_flag or rflag
     return {"accept": acc, "acc_flag": aflag, "n_accept": n, "n_flag": n_flag,
             "out_tokens": out, "tok_flag": tok_flag, "target_argmax": targmax}
 
@@ -400,7 +444,8 @@ def confidence_verify(draft, target, tokens, P: Params, seed=0, iteration=0,
                       k_row=None, seqs=None):
     """Full iteration: confidence signals, k_next, verification, correction.
 
-    draft, target: float64 [B, K, V]; tokens: int [B, K].
+    draft: float64 [B, K, V]; target: float64 [B, K, V], or [B, K + 1, V]
+    with P.bonus; tokens: int [B, K].
     seqs: optional list of sequence indices to evaluate (others left empty).
     """
     draft = np.asarray(draft, dtype=np.float64)
@@ -415,7 +460,7 @@ def confidence_verify(draft, target, tokens, P: Params, seed=0, iteration=0,
     res.acc_flag = np.zeros((B, K), dtype=bool)
     res.n_accept = np.full(B, -1, dtype=np.int64)
     res.n_flag = np.zeros(B, dtype=bool)
-    res.out_tokens = np.full((B, K), -1, dtype=np.int64)
+    res.out_tokens = np.full((B, K + 1 if P.bonus else K), -1, dtype=np.int64)
     res.tok_flag = np.zeros(B, dtype=bool)
     res.target_argmax = np.full((B, K), -1, dtype=np.int64)
     for b in seq_list:
@@ -439,7 +484,8 @@ def verify(draft, target, tokens, conf, P: Params, seed=0, iteration=0, k_row=No
     kb = _k_rows(B, K, k_row)
     out = {"accept": np.zeros((B, K), dtype=bool), "acc_flag": np.zeros((B, K), dtype=bool),
            "n_accept": np.zeros(B, dtype=np.int64), "n_flag": np.zeros(B, dtype=bool),
-           "out_tokens": np.full((B, K), -1, dtype=np.int64), "tok_flag": np.zeros(B, dtype=bool)}
+           "out_tokens": np.full((B, K + 1 if P.bonus else K), -1, dtype=np.int64),
+           "tok_flag": np.zeros(B, dtype=bool)}
     for b in range(B):
         k_b = int(kb[b])
         v = verify_sequence(draft[b], target[b], tokens[b], conf[b], k_b, P, seed, b, iteration)
@@ -460,7 +506,8 @@ def decode_sim_sequence(gen_rows, b, iterations, K_max, P: Params, seed):
     """Replay the draft-length / acceptance trajectory of sequence b.
 
     gen_rows(it, b, k) -> (draft[k, V], target[k, V], tokens[k]) supplies the
-    drafted positions present at iteration it (float arrays).  The first
+    drafted positions present at iteration it (float arrays; with P.bonus the
+    target has k + 1 rows, the last being the bonus row).  The first
     iteration drafts K_max positions; each later one drafts the k chosen from
     the previous iteration's confidence (reading C4).  Returns a list of dicts
     (k, n_accept, k_next, out_tokens, flagged) per iteration; `flagged` marks
@@ -482,9 +529,9 @@ def decode_sim_sequence(gen_rows, b, iterations, K_max, P: Params, seed):
         toks = np.full(K_max, -1, dtype=np.int64)
         toks[:k] = tok
         dd = np.zeros((K_max, V))
-        tt = np.zeros((K_max, V))
+        tt = np.zeros((K_max + 1 if P.bonus else K_max, V))
         dd[:k] = d
-        tt[:k] = t
+        tt[:t.shape[0]] = t
         v = verify_sequence(dd, tt, toks, np.concatenate([conf, np.zeros(K_max - k)]), k, P,
                             seed, b, it)
         traj.append({"k": k, "n_accept": v["n_accept"], "k_next": k_next,

@@ -412,3 +412,78 @@ def test_decode_sim_replay_feeds_k_forward():
         assert b["k"] == a["k_next"]
     for s in traj:
         assert 1 <= s["k_next"] <= 16 and 0 <= s["n_accept"] <= s["k"]
+
+
+# ---------------------------------------------------------------- fixed k, bonus row
+
+def test_fixed_draft_length_ignores_confidence():
+    # Table III, "fixed k": the draft length no longer follows the confidence
+    pp = P(k_max=16, k_min=2, k_fixed=9)
+    for window in ([0.0] * 4, [1.0] * 4, [0.3, 0.9], []):
+        assert O.next_draft_length(window, pp) == (9, False)
+
+
+def test_bonus_argmax_by_sorting():
+    rng = np.random.default_rng(30)
+    for _ in range(20):
+        z = np.round(rng.normal(0, 1, 50), 1)          # ties are common at one decimal
+        tok, flag = O.bonus_token(z, "paper", 0, 0, 0, 0)
+        top = max(z)
+        assert tok == min(i for i in range(50) if z[i] == top) and not flag
+
+
+@pytest.mark.parametrize("V", [8, 100])
+def test_bonus_draw_has_the_verifier_law(V):
+    # the sampled bonus token is the two-level race with r = p: its law is p
+    # (V = 100 spans four groups of 32, the last one partial)
+    rng = np.random.default_rng(31 + V)
+    zt = rng.normal(0, 1.0, V)
+    p = sps.softmax(zt)
+    n = 20000
+    counts = np.zeros(V)
+    for it in range(n):
+        tok, _ = O.bonus_token(zt, "sampled", 5, 3, 4, it)
+        counts[tok] += 1
+    if V == 8:
+        chi2 = ((counts - p * n) ** 2 / (p * n)).sum()
+        assert st.chi2.sf(chi2, V - 1) > 1e-3
+    else:
+        G = O.philox.GROUP
+        gm = np.array([p[i:i + G].sum() for i in range(0, V, G)]) * n
+        gc = np.array([counts[i:i + G].sum() for i in range(0, V, G)])
+        assert st.chi2.sf(((gc - gm) ** 2 / gm).sum(), len(gm) - 1) > 1e-3
+        top = np.argsort(-p)[:8]
+        e = p[top] * n
+        assert st.chi2.sf(((counts[top] - e) ** 2 / e).sum(), len(top)) > 1e-4
+
+
+def test_bonus_row_follows_an_accepted_window():
+    # K = 1, tau = 0, the verifier's extra row present: when the draft is
+    # accepted the second emitted token follows the extra row's law p1; when
+    # it is rejected only the correction is emitted (no bonus)
+    rng = np.random.default_rng(33)
+    V = 8
+    zt, zd = _rows8(rng, V)
+    z1 = rng.normal(0, 1.0, V)
+    p1 = sps.softmax(z1)
+    pp = P(k_max=1, rule="sampled", beta_rank=0, tau_base=0.0, gamma=0.0, bonus=True)
+    n = 6000
+    xs = rng.choice(V, size=n, p=sps.softmax(zd))
+    counts = np.zeros(V)
+    for it in range(n):
+        v = O.verify_sequence(zd[None], np.stack([zt, z1]), np.array([xs[it]]), np.array([0.5]), 1, pp, 78, 0, it)
+        out = v["out_tokens"]
+        assert out.shape == (2,)
+        if v["n_accept"] == 1:
+            assert out[0] == xs[it] and 0 <= out[1] < V
+            counts[out[1]] += 1
+        else:
+            assert out[1] == -1
+    m = counts.sum()
+    assert m > 1000
+    chi2 = ((counts - p1 * m) ** 2 / (p1 * m)).sum()
+    assert st.chi2.sf(chi2, V - 1) > 1e-3
+    # PAPER rule: the bonus token is the extra row's argmax
+    pq = P(k_max=1, rule="paper", beta_rank=0, tau_base=100.0, gamma=0.0, bonus=True)
+    v = O.verify_sequence(zd[None], np.stack([zt, z1]), np.array([0]), np.array([0.5]), 1, pq, 0, 0, 0)
+    assert v["n_accept"] == 1 and v["out_tokens"][1] == int(np.argmax(z1))
