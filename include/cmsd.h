@@ -26,7 +26,11 @@
  *   - Return value: CMSD_OK, or a negative cmsd_status.  Argument errors are
  *     detected on the host before anything is enqueued.  Errors that only the
  *     device can see (a drafted token outside [0, V), k_row outside [0, K]) are
- *     clamped and recorded in the workspace; cmsd_workspace_errors reads them.
+ *     clamped before any load and recorded in the workspace;
+ *     cmsd_workspace_errors reads them.
+ *   - Calls that draw a residual token (CMSD_RULE_SAMPLED) or use the bonus row
+ *     launch a second kernel after the streaming kernel, on the same stream,
+ *     which makes a second pass over one row of each sequence that needs it.
  *   - Logits must be finite or -inf (masked vocabulary entries, probability 0);
  *     |logit| < 1e29; every row needs at least one finite logit.  +inf and NaN
  *     give unspecified results.
@@ -81,11 +85,41 @@ typedef struct {
   int32_t tau_sign;       /* +1: tau_t = tau_base + gamma (1 - C_t), the printed
                              equation; -1: tau_base + gamma C_t, the prose reading */
   int32_t rule;           /* cmsd_rule */
+  int32_t k_fixed;        /* 0: adaptive draft length; k_min <= k_fixed <= k_max: the
+                             next draft length is this constant (the fixed-k variants
+                             of the ablation, Sec. IV, Table III) */
+  int32_t bonus;          /* 1: the verifier scores one more position than was drafted
+                             (Sec. III.A(2): the verifier's own prediction follows the
+                             accepted prefix).  target_logits is then [B][K+1][V] (row
+                             k_row[b] of sequence b is that extra row) and out_tokens is
+                             [B][K+1]; when all k_row[b] drafts are accepted, slot
+                             k_row[b] receives the extra row's argmax (PAPER rule) or a
+                             draw from its softmax (SAMPLED rule).  Requires V * dtype
+                             size to be a multiple of 16 bytes.  0: no extra row. */
 } cmsd_params;
 
 /* Defaults: k_min 1, k_max K, lambda 1/3 each, beta_sig 1, beta_rank 3 (PAPER)
- * or 0 (SAMPLED), alpha 1, tau_base 0.1, gamma 1, tau_sign +1. */
+ * or 0 (SAMPLED), alpha 1, tau_base 0.1, gamma 1, tau_sign +1, k_fixed 0,
+ * bonus 0. */
 void cmsd_params_default(cmsd_params* p, int K, int rule);
+
+/* The variants of the ablation (Sec. IV, Table III) as parameter sets:
+ * the defaults above, then
+ *   FIXED_K       k_fixed = k_max (fixed draft length, adaptive tau)
+ *   FIXED_TAU     gamma = 0 (adaptive draft length, fixed tau = tau_base)
+ *   FIXED_K_TAU   both (no confidence modulation)
+ *   ENTROPY_ONLY, MARGIN_ONLY, SOFTMAX_ONLY   lambda one-hot.
+ * Returns CMSD_EINVAL for an unknown preset. */
+typedef enum {
+  CMSD_PRESET_FULL = 0,
+  CMSD_PRESET_FIXED_K = 1,
+  CMSD_PRESET_FIXED_TAU = 2,
+  CMSD_PRESET_FIXED_K_TAU = 3,
+  CMSD_PRESET_ENTROPY_ONLY = 4,
+  CMSD_PRESET_MARGIN_ONLY = 5,
+  CMSD_PRESET_SOFTMAX_ONLY = 6
+} cmsd_preset;
+int cmsd_params_preset(cmsd_params* p, int K, int rule, int preset);
 
 /* Bytes of workspace a call with these sizes needs on the current device.
  * The workspace must be zeroed once (cmsd_workspace_init) before first use;
@@ -94,8 +128,8 @@ size_t cmsd_workspace_bytes(int B, int K, int V);
 int cmsd_workspace_init(void* ws, size_t ws_bytes, void* stream);
 
 /* Device-detected input errors since the last init/read (bit 0: drafted token
- * out of range, bit 1: k_row out of range, bit 2: workspace shared by calls
- * that were not ordered on one stream); clears them.  Synchronises `stream`. */
+ * out of range, bit 1: k_row out of range); clears them.  Synchronises
+ * `stream`. */
 int cmsd_workspace_errors(void* ws, size_t ws_bytes, void* stream, uint32_t* flags_out);
 
 /*
@@ -128,11 +162,13 @@ int cmsd_confidence(const void* draft_logits, int B, int K, int V, int dtype,
  *   uniform counter (g>>2, b, n, iteration<<2 | 2) word g&3 and the group with
  *   the least -log(1-U_g) / R_g wins (R_g its residual mass); entry v of that
  *   group gets counter (v>>2, b, n, iteration<<2 | 1) word v&3 and the least
- *   -log(1-U_v) / r_v wins.  The token's law is r_v / sum(r).
+ *   -log(1-U_v) / r_v wins.  The token's law is r_v / sum(r).  The bonus token
+ *   (SAMPLED rule) is the same race over p of the extra row, with n = k_row[b].
  * Outputs: n_accept [B] (first rejected position, k_row[b] if none);
- *   out_tokens [B][K]: accepted drafts, then the correction at n_accept (when
- *   n_accept < k_row[b]), then -1; accept [B][K] (uint8, 0 beyond k_row) may be
- *   NULL.
+ *   out_tokens [B][K] ([B][K+1] with the bonus row): accepted drafts, then the
+ *   correction at n_accept (when n_accept < k_row[b]) or the bonus token (when
+ *   n_accept == k_row[b] and p->bonus), then -1; accept [B][K] (uint8, 0
+ *   beyond k_row) may be NULL.
  */
 int cmsd_verify(const void* draft_logits, const void* target_logits,
                 const int32_t* draft_tokens, const int32_t* k_row,
@@ -144,9 +180,10 @@ int cmsd_verify(const void* draft_logits, const void* target_logits,
 
 /*
  * The fused pass: cmsd_confidence and cmsd_verify in one streaming read of
- * both logit tensors (plus, in SAMPLED mode, a second pass over the rejected
- * row pair of each sequence only).  Same arguments and outputs as the two
- * calls above; n_accept and out_tokens are required, the rest may be NULL.
+ * both logit tensors (plus a second pass over the rejected row pair, or the
+ * bonus row, of each sequence that needs one).  Same arguments
+ * and outputs as the two calls above; n_accept and out_tokens are required,
+ * the rest may be NULL.
  */
 int cmsd_confidence_verify(const void* draft_logits, const void* target_logits,
                            const int32_t* draft_tokens, const int32_t* k_row,
@@ -166,9 +203,10 @@ int cmsd_confidence_verify(const void* draft_logits, const void* target_logits,
  * It allocates nothing.
  *   - Arguments and outputs: as cmsd_confidence_verify, minus ws / ws_bytes.
  *   - Limit: a problem whose cmsd_workspace_bytes(B, K, V) exceeds
- *     CMSD_STATIC_SCRATCH_BYTES (4 MiB; on a 152-SM GB300 that admits B*K up
- *     to about 41,000 positions for K >= 8, 26,000 at K = 1) is rejected with
- *     CMSD_ESCRATCH before anything is enqueued.
+ *     CMSD_STATIC_SCRATCH_BYTES (4 MiB; on a 152-SM GB300 at V = 128256 that
+ *     admits about 1,000 sequences of K = 8, and B*K up to about 20,000
+ *     positions at V = 32000) is rejected with CMSD_ESCRATCH, after the other
+ *     argument checks and before anything is enqueued.
  *   - Each call first zero-fills, on `stream`, the part of the scratch that
  *     its layout uses, so device-side error flags (cmsd_workspace_errors) of
  *     an earlier call are not kept; use cmsd_confidence_verify with a caller
@@ -202,11 +240,14 @@ int cmsd_philox_fill(uint64_t seed, uint32_t c0, uint32_t c1, uint32_t c2, uint3
 
 /* Kernel timing: while enabled, each cmsd_confidence / cmsd_verify /
  * cmsd_confidence_verify call records CUDA events on its stream around its
- * streaming kernel and around its residual-resample kernel (SAMPLED rule),
- * for up to max_calls calls.  cmsd_profile_stop synchronises those events and
- * writes, per call, the streaming-kernel time and the resample-kernel time in
- * milliseconds (0 when there was none); either array may be NULL; *n_out
- * receives the number of calls recorded.  Not thread-safe. */
+ * streaming kernel and around its resample kernel (sampled rule or bonus
+ * row), for up to max_calls calls.  cmsd_profile_stop synchronises those
+ * events and writes, per call, the streaming-kernel time and the
+ * resample-kernel time in milliseconds (0 when there was none); either array
+ * may be NULL; *n_out receives the number of calls recorded.  An event
+ * between the two kernels keeps the second from starting during the first's
+ * tail, so timed calls run a little slower than untimed ones.
+ * Not thread-safe. */
 int cmsd_profile_start(int max_calls);
 int cmsd_profile_stop(float* stream_ms, float* resample_ms, int max_out, int* n_out);
 

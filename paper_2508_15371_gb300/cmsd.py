@@ -35,13 +35,16 @@ class Params(ctypes.Structure):
         ("gamma", ctypes.c_float),
         ("tau_sign", ctypes.c_int32),
         ("rule", ctypes.c_int32),
+        ("k_fixed", ctypes.c_int32),
+        ("bonus", ctypes.c_int32),
     ]
 
     def as_dict(self):
         return dict(k_min=self.k_min, k_max=self.k_max, lam=tuple(float(x) for x in self.lam),
                     beta_sig=float(self.beta_sig), beta_rank=self.beta_rank, alpha=float(self.alpha),
                     tau_base=float(self.tau_base), gamma=float(self.gamma), tau_sign=self.tau_sign,
-                    rule="sampled" if self.rule == RULE_SAMPLED else "paper")
+                    rule="sampled" if self.rule == RULE_SAMPLED else "paper", k_fixed=self.k_fixed,
+                    bonus=bool(self.bonus))
 
 
 class CmsdError(RuntimeError):
@@ -53,6 +56,7 @@ _lib_lock = threading.Lock()
 
 _SIGS = {
     "cmsd_params_default": (None, [_vp, _c_int, _c_int]),
+    "cmsd_params_preset": (_c_int, [_vp, _c_int, _c_int, _c_int]),
     "cmsd_workspace_bytes": (_c_sz, [_c_int, _c_int, _c_int]),
     "cmsd_workspace_init": (_c_int, [_vp, _c_sz, _vp]),
     "cmsd_workspace_errors": (_c_int, [_vp, _c_sz, _vp, ctypes.POINTER(ctypes.c_uint32)]),
@@ -102,21 +106,28 @@ def _check(rc, what):
         raise CmsdError(f"{what}: {msg} [{rc}]")
 
 
-def params(K, rule="paper", **kw):
-    """Default cmsd_params for window K and rule ('paper' or 'sampled'), then overrides.
+PRESETS = {"full": 0, "fixed_k": 1, "fixed_tau": 2, "fixed_k_tau": 3, "entropy_only": 4,
+           "margin_only": 5, "softmax_only": 6}
+
+
+def params(K, rule="paper", preset="full", **kw):
+    """cmsd_params for window K, rule ('paper' or 'sampled') and ablation
+    preset (PRESETS: the variants of Table III), then overrides.
 
     Keyword names: k_min, k_max, lam (3-tuple), beta_sig, beta_rank, alpha,
-    tau_base, gamma, tau_sign.
+    tau_base, gamma, tau_sign, k_fixed, bonus.
     """
     r = RULE_SAMPLED if rule in ("sampled", RULE_SAMPLED) else RULE_PAPER
     p = Params()
-    lib().cmsd_params_default(ctypes.byref(p), int(K), r)
+    _check(lib().cmsd_params_preset(ctypes.byref(p), int(K), r, PRESETS[preset]), "cmsd_params_preset")
     for k, v in kw.items():
         if k == "lam":
             for j in range(3):
                 p.lam[j] = float(v[j])
         elif k == "rule":
             p.rule = RULE_SAMPLED if v in ("sampled", RULE_SAMPLED) else RULE_PAPER
+        elif k == "bonus":
+            p.bonus = 1 if v else 0
         else:
             setattr(p, k, v)
     return p
@@ -138,6 +149,13 @@ def _dtype_code(t):
     if t.dtype == torch.bfloat16:
         return BF16
     raise CmsdError(f"logits must be float32 or bfloat16, got {t.dtype}")
+
+
+def _check_target(draft, target, p):
+    B, K, V = draft.shape
+    want = (B, K + 1, V) if p.bonus else (B, K, V)
+    if draft.dtype != target.dtype or tuple(target.shape) != want:
+        raise CmsdError(f"target logits must be {want} of the drafter's dtype, got {tuple(target.shape)}")
 
 
 def _stream():
@@ -215,9 +233,10 @@ def verify(draft, target, tokens, conf, draft_lse=None, k_row=None, p=None, seed
     _need_cuda(draft, target, tokens, conf, draft_lse, k_row)
     B, K, V = draft.shape
     p = p if p is not None else params(K)
+    _check_target(draft, target, p)
     dev = draft.device
     o = {"n_accept": _out(out, "n_accept", (B,), torch.int32, dev),
-         "out_tokens": _out(out, "out_tokens", (B, K), torch.int32, dev),
+         "out_tokens": _out(out, "out_tokens", (B, K + 1 if p.bonus else K), torch.int32, dev),
          "accept": _out(out, "accept", (B, K), torch.uint8, dev)}
     ws = ws if ws is not None else workspace(B, K, V)
     rc = lib().cmsd_verify(_ptr(draft), _ptr(target), _ptr(tokens), _ptr(k_row), B, K, V,
@@ -234,10 +253,9 @@ def confidence_verify(draft, target, tokens, k_row=None, p=None, seed=0, iterati
     H, margin, argmax, conf, lse."""
     torch = _torch()
     _need_cuda(draft, target, tokens, k_row)
-    if draft.dtype != target.dtype or draft.shape != target.shape:
-        raise CmsdError("draft and target logits must have the same shape and dtype")
     B, K, V = draft.shape
     p = p if p is not None else params(K)
+    _check_target(draft, target, p)
     dev = draft.device
     o = {}
     for n in ("H", "margin", "conf", "lse"):
@@ -245,7 +263,7 @@ def confidence_verify(draft, target, tokens, k_row=None, p=None, seed=0, iterati
     o["argmax"] = _out(out, "argmax", (B, K), torch.int32, dev, signals)
     o["k_next"] = _out(out, "k_next", (B,), torch.int32, dev)
     o["n_accept"] = _out(out, "n_accept", (B,), torch.int32, dev)
-    o["out_tokens"] = _out(out, "out_tokens", (B, K), torch.int32, dev)
+    o["out_tokens"] = _out(out, "out_tokens", (B, K + 1 if p.bonus else K), torch.int32, dev)
     o["accept"] = _out(out, "accept", (B, K), torch.uint8, dev, signals)
     ws = ws if ws is not None else workspace(B, K, V)
     rc = lib().cmsd_confidence_verify(
@@ -265,10 +283,9 @@ def confidence_verify_static(draft, target, tokens, k_row=None, p=None, seed=0, 
     not allocate passes them all.  Calls on one device must not overlap."""
     torch = _torch()
     _need_cuda(draft, target, tokens, k_row)
-    if draft.dtype != target.dtype or draft.shape != target.shape:
-        raise CmsdError("draft and target logits must have the same shape and dtype")
     B, K, V = draft.shape
     p = p if p is not None else params(K)
+    _check_target(draft, target, p)
     dev = draft.device
     o = {}
     for n in ("H", "margin", "conf", "lse"):
@@ -276,7 +293,7 @@ def confidence_verify_static(draft, target, tokens, k_row=None, p=None, seed=0, 
     o["argmax"] = _out(out, "argmax", (B, K), torch.int32, dev, signals)
     o["k_next"] = _out(out, "k_next", (B,), torch.int32, dev)
     o["n_accept"] = _out(out, "n_accept", (B,), torch.int32, dev)
-    o["out_tokens"] = _out(out, "out_tokens", (B, K), torch.int32, dev)
+    o["out_tokens"] = _out(out, "out_tokens", (B, K + 1 if p.bonus else K), torch.int32, dev)
     o["accept"] = _out(out, "accept", (B, K), torch.uint8, dev, signals)
     rc = lib().cmsd_confidence_verify_static(
         _ptr(draft), _ptr(target), _ptr(tokens), _ptr(k_row), B, K, V, _dtype_code(draft),
@@ -303,7 +320,8 @@ def profile_start(max_calls):
 
 
 def profile_stop(max_calls):
-    """Per-call (streaming-kernel ms, resample-kernel ms) recorded since profile_start."""
+    """Per-call (streaming-kernel ms, resample-kernel ms) recorded since profile_start
+    (the second is 0 for calls without a resample kernel)."""
     a = (ctypes.c_float * max(1, max_calls))()
     b = (ctypes.c_float * max(1, max_calls))()
     n = ctypes.c_int(0)
@@ -348,7 +366,7 @@ class FusedCall:
         o.setdefault("accept", torch.empty((B, K), dtype=torch.uint8, device=dev) if signals else None)
         o.setdefault("k_next", torch.empty((B,), dtype=torch.int32, device=dev))
         o.setdefault("n_accept", torch.empty((B,), dtype=torch.int32, device=dev))
-        o.setdefault("out_tokens", torch.empty((B, K), dtype=torch.int32, device=dev))
+        o.setdefault("out_tokens", torch.empty((B, K + 1 if p.bonus else K), dtype=torch.int32, device=dev))
         self.out = o
         self.ws = ws if ws is not None else workspace(B, K, V)
         self._keep = (draft, target, tokens, k_row, p)

@@ -27,8 +27,8 @@ int cuda_fail(cudaError_t e) {
 
 std::mutex g_mu;
 std::map<int, int> g_sms;                                   // device -> SM count
-std::map<std::tuple<int, int, int, int, int>, int> g_occ;   // (dev, dtype, mode, sampled, smem) -> blocks/SM
-std::map<std::pair<int, int>, int> g_occ_res;               // (dev, dtype) -> blocks/SM
+std::map<std::tuple<int, int, int, int, int>, int> g_occ;   // (dev, dtype, mode, variant, smem) -> blocks/SM
+std::map<std::tuple<int, int, int>, int> g_occ_res;          // (dev, dtype, sampled) -> blocks/SM
 
 int device_sms(int* sms) {
   int dev = 0;
@@ -46,18 +46,19 @@ int device_sms(int* sms) {
   return CMSD_OK;
 }
 
-int stream_grid(int dtype, int mode, bool sampled, size_t smem, int* grid) {
+int stream_grid(int dtype, int mode, bool sampled, bool second, size_t smem, int* grid) {
   int sms = 0;
   int rc = device_sms(&sms);
   if (rc) return rc;
   int dev = 0;
   cudaGetDevice(&dev);
-  const auto key = std::make_tuple(dev, dtype, mode, sampled ? 1 : 0, (int)smem);
+  const int variant = (sampled ? 1 : 0) | (second ? 2 : 0);
+  const auto key = std::make_tuple(dev, dtype, mode, variant, (int)smem);
   std::lock_guard<std::mutex> lk(g_mu);
   auto it = g_occ.find(key);
   if (it == g_occ.end()) {
     int nb = 0;
-    cudaError_t e = occupancy_stream(dtype, mode, sampled, smem, &nb);
+    cudaError_t e = occupancy_stream(dtype, mode, sampled, second, smem, &nb);
     if (e != cudaSuccess) return cuda_fail(e);
     if (nb < 1) nb = 1;
     it = g_occ.emplace(key, nb).first;
@@ -66,18 +67,18 @@ int stream_grid(int dtype, int mode, bool sampled, size_t smem, int* grid) {
   return CMSD_OK;
 }
 
-int resample_grid(int dtype, int* grid) {
+int resample_grid(int dtype, bool sampled, int* grid) {
   int sms = 0;
   int rc = device_sms(&sms);
   if (rc) return rc;
   int dev = 0;
   cudaGetDevice(&dev);
+  const auto key = std::make_tuple(dev, dtype, sampled ? 1 : 0);
   std::lock_guard<std::mutex> lk(g_mu);
-  auto key = std::make_pair(dev, dtype);
   auto it = g_occ_res.find(key);
   if (it == g_occ_res.end()) {
     int nb = 0;
-    cudaError_t e = occupancy_resample(dtype, &nb);
+    cudaError_t e = occupancy_resample(dtype, sampled, &nb);
     if (e != cudaSuccess) return cuda_fail(e);
     if (nb < 1) nb = 1;
     it = g_occ_res.emplace(key, nb).first;
@@ -92,30 +93,32 @@ constexpr size_t kAlign = 256;
 size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
-  size_t err, row_done, seq_done, res_done, rej_count, res_cta_done;
-  size_t rej, row_conf, row_acc, row_targmax, row_dstat, row_tstat, part, rpart;
+  size_t err, row_done, seq_word, seq_done, rec_count, res_cta_done, res_done;
+  size_t rec, row_conf, row_acc, row_targmax, row_dstat, row_tstat, part, rpart;
   size_t total;
 };
 
-// The error word sits at offset 0 so that cmsd_workspace_errors needs no sizes.
+// The error word sits at offset 0 so that cmsd_workspace_errors needs no sizes;
+// the two queue counters follow it (offsets 256 and 512).
 Layout make_layout(int B, int K, int wmax) {
   Layout L;
   const size_t BK = (size_t)B * (size_t)K;
   size_t o = 0;
   L.err = o; o += up(sizeof(unsigned));
+  L.rec_count = o; o += up(sizeof(int));
+  L.res_cta_done = o; o += up(sizeof(int));
   L.row_done = o; o += up(BK * sizeof(int));
+  L.seq_word = o; o += up((size_t)B * sizeof(unsigned long long));
   L.seq_done = o; o += up((size_t)B * sizeof(int));
   L.res_done = o; o += up((size_t)B * sizeof(int));
-  L.rej_count = o; o += up(sizeof(int));
-  L.res_cta_done = o; o += up(sizeof(int));
-  L.rej = o; o += up((size_t)B * sizeof(RejRec));
-  L.row_conf = o; o += up(BK * sizeof(float));
+  L.rec = o; o += up((size_t)B * sizeof(int4));
+  L.row_conf = o; o += up(BK * sizeof(unsigned long long));
   L.row_acc = o; o += up(BK * sizeof(int));
   L.row_targmax = o; o += up(BK * sizeof(int));
   L.row_dstat = o; o += up(BK * sizeof(float2));
   L.row_tstat = o; o += up(BK * sizeof(float2));
   L.part = o; o += up((BK + (size_t)wmax) * sizeof(Partial));
-  L.rpart = o; o += up(((size_t)B + (size_t)wmax) * sizeof(RacePartial));
+  L.rpart = o; o += up(((size_t)B + (size_t)wmax) * sizeof(UnitResult));
   L.total = o;
   return L;
 }
@@ -125,18 +128,19 @@ Workspace carve(void* ws, const Layout& L) {
   Workspace W;
   W.err = (unsigned*)(p + L.err);
   W.row_done = (int*)(p + L.row_done);
+  W.seq_word = (unsigned long long*)(p + L.seq_word);
   W.seq_done = (int*)(p + L.seq_done);
-  W.res_done = (int*)(p + L.res_done);
-  W.rej_count = (int*)(p + L.rej_count);
+  W.rec_count = (int*)(p + L.rec_count);
   W.res_cta_done = (int*)(p + L.res_cta_done);
-  W.rej = (RejRec*)(p + L.rej);
-  W.row_conf = (float*)(p + L.row_conf);
+  W.res_done = (int*)(p + L.res_done);
+  W.rec = (int4*)(p + L.rec);
+  W.row_conf = (unsigned long long*)(p + L.row_conf);
   W.row_acc = (int*)(p + L.row_acc);
   W.row_targmax = (int*)(p + L.row_targmax);
   W.row_dstat = (float2*)(p + L.row_dstat);
   W.row_tstat = (float2*)(p + L.row_tstat);
   W.part = (Partial*)(p + L.part);
-  W.rpart = (RacePartial*)(p + L.rpart);
+  W.rpart = (UnitResult*)(p + L.rpart);
   return W;
 }
 
@@ -154,7 +158,7 @@ struct Profiler {
   bool on = false;
   int max_calls = 0;
   int n = 0;
-  std::vector<cudaEvent_t> ev;   // 3 per call: start, after stream kernel, after resample
+  std::vector<cudaEvent_t> ev;   // 3 per call: start, after the streaming kernel, after the resample kernel
 } g_prof;
 
 void prof_record(int slot, cudaStream_t s) {
@@ -191,7 +195,18 @@ int check_params(const cmsd_params* p, bool need_rule) {
   if (!(p->alpha > 0.f && p->alpha <= 1.f)) return CMSD_EINVAL;
   if (!isfinite(p->tau_base) || !isfinite(p->gamma)) return CMSD_EINVAL;
   if (p->tau_sign != 1 && p->tau_sign != -1) return CMSD_EINVAL;
+  if (p->k_fixed != 0 && (p->k_fixed < p->k_min || p->k_fixed > p->k_max)) return CMSD_EINVAL;
+  if (p->bonus != 0 && p->bonus != 1) return CMSD_EINVAL;
   return CMSD_OK;
+}
+
+// With the bonus row the verifier tensor has K + 1 rows per sequence while the
+// drafter's has K: their rows stay equally aligned only if a row is a whole
+// number of 16-byte vectors.
+int check_bonus_layout(const cmsd_params* p, int V, int dtype) {
+  if (!p->bonus) return CMSD_OK;
+  const size_t row_bytes = (size_t)V * (dtype == CMSD_F32 ? 4 : 2);
+  return (row_bytes % 16) == 0 ? CMSD_OK : CMSD_EINVAL;
 }
 
 void fill_params(StreamArgs& a, const cmsd_params* p) {
@@ -206,6 +221,14 @@ void fill_params(StreamArgs& a, const cmsd_params* p) {
   a.tau_base = p->tau_base;
   a.gamma = p->gamma;
   a.tau_sign = p->tau_sign;
+  a.k_fixed = p->k_fixed;
+  a.bonus = p->bonus;
+}
+
+void fill_sizes(StreamArgs& a, int B, int K, int V) {
+  a.B = B; a.K = K; a.V = V;
+  a.inv_log_v = (float)(1.0 / log((double)V));
+  a.soft_norm = (float)(1.0 / (1.0 - 1.0 / (double)V));
 }
 
 int launch(int dtype, int mode, bool sampled, StreamArgs& a, void* ws, size_t ws_bytes,
@@ -216,24 +239,36 @@ int launch(int dtype, int mode, bool sampled, StreamArgs& a, void* ws, size_t ws
   const Layout L = make_layout(a.B, a.K, wmax);
   if (!ws || ws_bytes < L.total) return CMSD_ENOWS;
   a.ws = carve(ws, L);
+  const bool bonus = mode != kModeConf && a.bonus;
+  a.Kt = bonus ? a.K + 1 : a.K;
+  a.Ko = bonus ? a.K + 1 : a.K;
+  const bool second = mode != kModeConf && (sampled || bonus);
   const size_t smem = stream_smem_bytes(a.B, a.k_row != nullptr);
   int grid = 0;
-  rc = stream_grid(dtype, mode, sampled, smem, &grid);
+  rc = stream_grid(dtype, mode, sampled, second, smem, &grid);
   if (rc) return rc;
+  int g2 = 0;
+  if (second) {
+    rc = resample_grid(dtype, sampled, &g2);
+    if (rc) return rc;
+  }
   a.nwarps = grid * kStreamWarps;
   prof_record(0, s);
-  cudaError_t e = dtype == CMSD_F32 ? launch_stream_f32(mode, sampled, a, grid, smem, s)
-                                    : launch_stream_bf16(mode, sampled, a, grid, smem, s);
+  cudaError_t e = dtype == CMSD_F32 ? launch_stream_f32(mode, sampled, second, a, grid, smem, s)
+                                    : launch_stream_bf16(mode, sampled, second, a, grid, smem, s);
   if (e != cudaSuccess) return cuda_fail(e);
   prof_record(1, s);
-  if (sampled && mode != kModeConf) {
-    int g2 = 0;
-    rc = resample_grid(dtype, &g2);
-    if (rc) return rc;
+  if (second) {
     StreamArgs b = a;
-    b.nwarps = g2 * kWarpsPerBlock;
-    e = dtype == CMSD_F32 ? launch_resample_f32(b, g2, s) : launch_resample_bf16(b, g2, s);
-    if (e != cudaSuccess) return cuda_fail(e);
+    b.nwarps = g2 * kResWarps;
+    e = dtype == CMSD_F32 ? launch_resample_f32(sampled, b, g2, s) : launch_resample_bf16(sampled, b, g2, s);
+    if (e != cudaSuccess) {
+      // the streaming kernel has queued rows that no resample kernel will
+      // drain: return the queue counters to zero so the workspace stays usable
+      cudaMemsetAsync(a.ws.rec_count, 0, sizeof(int), s);
+      cudaMemsetAsync(a.ws.res_cta_done, 0, sizeof(int), s);
+      return cuda_fail(e);
+    }
   }
   prof_record(2, s);
   return CMSD_OK;
@@ -246,6 +281,28 @@ StreamArgs blank_args() {
 }
 
 }  // namespace
+
+namespace cmsd {
+
+// Every host-side check of cmsd_confidence_verify (sizes, parameters, bonus
+// layout, required pointers, alignment), without launching anything.
+int validate_fused(const void* draft_logits, const void* target_logits, const int32_t* draft_tokens,
+                   const int32_t* k_row, int B, int K, int V, int dtype, const void* params,
+                   const int32_t* n_accept, const int32_t* out_tokens) {
+  const cmsd_params* p = (const cmsd_params*)params;
+  int rc = check_sizes(B, K, V, dtype, k_row);
+  if (rc) return rc;
+  rc = check_params(p, true);
+  if (rc) return rc;
+  rc = check_bonus_layout(p, V, dtype);
+  if (rc) return rc;
+  if (B == 0 || K == 0) return CMSD_OK;
+  if (!draft_logits || !target_logits || !draft_tokens || !n_accept || !out_tokens) return CMSD_EINVAL;
+  if (!aligned16(draft_logits) || !aligned16(target_logits)) return CMSD_EALIGN;
+  return CMSD_OK;
+}
+
+}  // namespace cmsd
 
 // ============================================================ C ABI
 
@@ -263,11 +320,28 @@ void cmsd_params_default(cmsd_params* p, int K, int rule) {
   p->gamma = 1.0f;
   p->tau_sign = 1;
   p->rule = rule;
+  p->k_fixed = 0;
+  p->bonus = 0;
+}
+
+int cmsd_params_preset(cmsd_params* p, int K, int rule, int preset) {
+  if (!p) return CMSD_EINVAL;
+  cmsd_params_default(p, K, rule);
+  switch (preset) {
+    case CMSD_PRESET_FULL: break;
+    case CMSD_PRESET_FIXED_K: p->k_fixed = p->k_max; break;
+    case CMSD_PRESET_FIXED_TAU: p->gamma = 0.0f; break;
+    case CMSD_PRESET_FIXED_K_TAU: p->k_fixed = p->k_max; p->gamma = 0.0f; break;
+    case CMSD_PRESET_ENTROPY_ONLY: p->lambda[0] = 1.0f; p->lambda[1] = p->lambda[2] = 0.0f; break;
+    case CMSD_PRESET_MARGIN_ONLY: p->lambda[1] = 1.0f; p->lambda[0] = p->lambda[2] = 0.0f; break;
+    case CMSD_PRESET_SOFTMAX_ONLY: p->lambda[2] = 1.0f; p->lambda[0] = p->lambda[1] = 0.0f; break;
+    default: return CMSD_EINVAL;
+  }
+  return CMSD_OK;
 }
 
 size_t cmsd_workspace_bytes(int B, int K, int V) {
-  (void)V;
-  if (B < 0 || K < 0) return 0;
+  if (B < 0 || K < 0 || V < 2) return 0;
   int wmax = 0;
   if (wmax_warps(&wmax)) return 0;
   return make_layout(B, K, wmax).total;
@@ -304,7 +378,7 @@ int cmsd_confidence(const void* draft_logits, int B, int K, int V, int dtype, co
   StreamArgs a = blank_args();
   a.draft = draft_logits;
   a.k_row = k_row;
-  a.B = B; a.K = K; a.V = V;
+  fill_sizes(a, B, K, V);
   fill_params(a, p);
   a.H = H; a.margin = margin; a.argmax = argmax; a.conf = conf; a.lse = lse; a.k_next = k_next;
   return launch(dtype, kModeConf, false, a, ws, ws_bytes, (cudaStream_t)stream);
@@ -319,6 +393,8 @@ int cmsd_verify(const void* draft_logits, const void* target_logits, const int32
   if (rc) return rc;
   rc = check_params(p, true);
   if (rc) return rc;
+  rc = check_bonus_layout(p, V, dtype);
+  if (rc) return rc;
   if (B == 0 || K == 0) return CMSD_OK;
   const bool sampled = p->rule == CMSD_RULE_SAMPLED;
   if (!draft_logits || !target_logits || !draft_tokens || !conf || !n_accept || !out_tokens)
@@ -330,7 +406,7 @@ int cmsd_verify(const void* draft_logits, const void* target_logits, const int32
   a.target = target_logits;
   a.tokens = draft_tokens;
   a.k_row = k_row;
-  a.B = B; a.K = K; a.V = V;
+  fill_sizes(a, B, K, V);
   fill_params(a, p);
   a.seed = seed;
   a.iteration = iteration;
@@ -346,20 +422,17 @@ int cmsd_confidence_verify(const void* draft_logits, const void* target_logits,
                            float* H, float* margin, int32_t* argmax, float* conf, float* lse,
                            int32_t* k_next, int32_t* n_accept, int32_t* out_tokens, uint8_t* accept,
                            void* ws, size_t ws_bytes, void* stream) {
-  int rc = check_sizes(B, K, V, dtype, k_row);
-  if (rc) return rc;
-  rc = check_params(p, true);
+  const int rc = validate_fused(draft_logits, target_logits, draft_tokens, k_row, B, K, V, dtype, p,
+                                n_accept, out_tokens);
   if (rc) return rc;
   if (B == 0 || K == 0) return CMSD_OK;
-  if (!draft_logits || !target_logits || !draft_tokens || !n_accept || !out_tokens) return CMSD_EINVAL;
-  if (!aligned16(draft_logits) || !aligned16(target_logits)) return CMSD_EALIGN;
   const bool sampled = p->rule == CMSD_RULE_SAMPLED;
   StreamArgs a = blank_args();
   a.draft = draft_logits;
   a.target = target_logits;
   a.tokens = draft_tokens;
   a.k_row = k_row;
-  a.B = B; a.K = K; a.V = V;
+  fill_sizes(a, B, K, V);
   fill_params(a, p);
   a.seed = seed;
   a.iteration = iteration;
@@ -407,12 +480,12 @@ int cmsd_profile_stop(float* stream_ms, float* resample_ms, int max_out, int* n_
   for (int j = 0; j < n; ++j) {
     cudaError_t e = cudaEventSynchronize(g_prof.ev[3 * j + 2]);
     if (e != cudaSuccess) return cuda_fail(e);
-    float a = 0.f, b = 0.f;
-    e = cudaEventElapsedTime(&a, g_prof.ev[3 * j], g_prof.ev[3 * j + 1]);
-    if (e == cudaSuccess) e = cudaEventElapsedTime(&b, g_prof.ev[3 * j + 1], g_prof.ev[3 * j + 2]);
+    float x = 0.f, y = 0.f;
+    e = cudaEventElapsedTime(&x, g_prof.ev[3 * j], g_prof.ev[3 * j + 1]);
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&y, g_prof.ev[3 * j + 1], g_prof.ev[3 * j + 2]);
     if (e != cudaSuccess) return cuda_fail(e);
-    if (stream_ms) stream_ms[j] = a;
-    if (resample_ms) resample_ms[j] = b;
+    if (stream_ms) stream_ms[j] = x;
+    if (resample_ms) resample_ms[j] = y;
   }
   if (n_out) *n_out = n;
   g_prof.n = 0;
@@ -424,7 +497,7 @@ int cmsd_launch_info(int dtype, int* warps_out, int* sms_out) {
   int sms = 0, grid = 0;
   int rc = device_sms(&sms);
   if (rc) return rc;
-  rc = stream_grid(dtype, kModeFused, true, stream_smem_bytes(0, false), &grid);
+  rc = stream_grid(dtype, kModeFused, true, true, stream_smem_bytes(0, false), &grid);
   if (rc) return rc;
   if (warps_out) *warps_out = grid * kStreamWarps;
   if (sms_out) *sms_out = sms;

@@ -1,6 +1,6 @@
 // Device primitives for sm_103a: fast base-2 exponential, packed bf16x2
-// min/max, packed f32x2 arithmetic, streaming loads, and the bulk-copy
-// (TMA) / mbarrier operations of the per-warp shared-memory pipelines.
+// min/max, packed f32x2 arithmetic, streaming loads and GPU-scope atomics
+// with acquire-release semantics.
 #pragma once
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -102,59 +102,10 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
   return r;
 }
 
-// ---- bulk copies and mbarriers --------------------------------------------
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
+__device__ __forceinline__ unsigned long long atom_add_acq_rel_u64(unsigned long long* p,
+                                                                   unsigned long long v) {
+  unsigned long long old;
+  asm volatile("atom.add.acq_rel.gpu.u64 %0, [%1], %2;" : "=l"(old) : "l"(p), "l"(v) : "memory");
+  return old;
 }
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void fence_mbar_init() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-__device__ __forceinline__ void fence_proxy_async() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("{\n\t.reg .b64 st;\n\tmbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n\t}"
-               ::"r"(bar), "r"(bytes) : "memory");
-}
-// global -> shared bulk copy of `bytes` (multiple of 16, both addresses 16-byte
-// aligned) completing on the mbarrier's transaction count
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-      ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
-}
-#ifndef CMSD_WAIT_HINT_NS
-#define CMSD_WAIT_HINT_NS 0
-#endif
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-#if CMSD_WAIT_HINT_NS > 0
-  asm volatile(
-      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity), "r"((uint32_t)CMSD_WAIT_HINT_NS)
-      : "memory");
-#else
-  asm volatile(
-      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-#endif
-  return ok != 0;
-}
-// Bounded wait: gives up after kWaitPolls polls (each poll may suspend the
-// thread for a short hardware-defined time) and reports failure.
-constexpr uint32_t kWaitPolls = 1u << 22;
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-  for (uint32_t it = 0; it < kWaitPolls; ++it)
-    if (mbar_try_wait(bar, parity)) return true;
-  return false;
-}
-
 }  // namespace cmsd

@@ -13,6 +13,7 @@
 #include <mutex>
 
 #include "cmsd.h"
+#include "cmsd_internal.h"
 
 namespace {
 
@@ -48,16 +49,16 @@ extern "C" int cmsd_confidence_verify_static(
     const int32_t* k_row, int B, int K, int V, int dtype, const cmsd_params* p, uint64_t seed,
     uint32_t iteration, float* H, float* margin, int32_t* argmax, float* conf, float* lse,
     int32_t* k_next, int32_t* n_accept, int32_t* out_tokens, uint8_t* accept, void* stream) {
-  if (B < 0 || K < 0) return CMSD_EINVAL;
-  if (B == 0 || K == 0)   // validates the other arguments, enqueues nothing
-    return cmsd_confidence_verify(draft_logits, target_logits, draft_tokens, k_row, B, K, V, dtype,
-                                  p, seed, iteration, H, margin, argmax, conf, lse, k_next,
-                                  n_accept, out_tokens, accept, nullptr, 0, stream);
+  // every argument check first: an invalid call enqueues nothing
+  int rc = cmsd::validate_fused(draft_logits, target_logits, draft_tokens, k_row, B, K, V, dtype, p,
+                                n_accept, out_tokens);
+  if (rc) return rc;
+  if (B == 0 || K == 0) return CMSD_OK;
   const size_t need = cmsd_workspace_bytes(B, K, V);
   if (need == 0) return CMSD_ECUDA;
   if (need > (size_t)CMSD_STATIC_SCRATCH_BYTES) return CMSD_ESCRATCH;
   void* ws = nullptr;
-  int rc = scratch_address(&ws);
+  rc = scratch_address(&ws);
   if (rc) return rc;
   if (cudaMemsetAsync(ws, 0, need, (cudaStream_t)stream) != cudaSuccess) return CMSD_ECUDA;
   return cmsd_confidence_verify(draft_logits, target_logits, draft_tokens, k_row, B, K, V, dtype,

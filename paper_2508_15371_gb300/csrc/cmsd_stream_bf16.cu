@@ -3,12 +3,19 @@
 
 namespace cmsd {
 
-cudaError_t launch_stream_bf16(int mode, bool sampled, const StreamArgs& a, int grid, size_t smem,
-                               cudaStream_t s) {
-  return launch_stream_t<uint16_t>(mode, sampled, a, grid, smem, s);
+cudaError_t launch_stream_bf16(int mode, bool sampled, bool second, const StreamArgs& a, int grid,
+                               size_t smem, cudaStream_t s) {
+  return launch_stream_t<uint16_t>(mode, sampled, second, a, grid, smem, s);
 }
-cudaError_t launch_resample_bf16(const StreamArgs& a, int grid, cudaStream_t s) {
-  return launch_resample_t<uint16_t>(a, grid, s);
+
+cudaError_t occupancy_stream_bf16(int mode, bool sampled, bool second, size_t smem, int* nb) {
+  return occupancy_stream_t<uint16_t>(mode, sampled, second, smem, nb);
 }
+
+cudaError_t launch_resample_bf16(bool sampled, const StreamArgs& a, int grid, cudaStream_t s) {
+  return launch_resample_t<uint16_t>(sampled, a, grid, s);
+}
+
+cudaError_t occupancy_resample_bf16(bool sampled, int* nb) { return occupancy_resample_t<uint16_t>(sampled, nb); }
 
 }  // namespace cmsd

@@ -4,20 +4,25 @@
 
 namespace cmsd {
 
-cudaError_t launch_stream_f32(int mode, bool sampled, const StreamArgs& a, int grid, size_t smem,
-                              cudaStream_t s) {
-  return launch_stream_t<float>(mode, sampled, a, grid, smem, s);
-}
-cudaError_t launch_resample_f32(const StreamArgs& a, int grid, cudaStream_t s) {
-  return launch_resample_t<float>(a, grid, s);
+cudaError_t occupancy_stream_bf16(int mode, bool sampled, bool second, size_t smem, int* nb);
+cudaError_t occupancy_resample_bf16(bool sampled, int* nb);
+
+cudaError_t launch_resample_f32(bool sampled, const StreamArgs& a, int grid, cudaStream_t s) {
+  return launch_resample_t<float>(sampled, a, grid, s);
 }
 
-cudaError_t occupancy_stream(int dtype, int mode, bool sampled, size_t smem, int* nb) {
-  return dtype == 0 ? occupancy_stream_t<float>(mode, sampled, smem, nb)
-                    : occupancy_stream_t<uint16_t>(mode, sampled, smem, nb);
+cudaError_t occupancy_resample(int dtype, bool sampled, int* nb) {
+  return dtype == 0 ? occupancy_resample_t<float>(sampled, nb) : occupancy_resample_bf16(sampled, nb);
 }
-cudaError_t occupancy_resample(int dtype, int* nb) {
-  return dtype == 0 ? occupancy_resample_t<float>(nb) : occupancy_resample_t<uint16_t>(nb);
+
+cudaError_t launch_stream_f32(int mode, bool sampled, bool second, const StreamArgs& a, int grid,
+                              size_t smem, cudaStream_t s) {
+  return launch_stream_t<float>(mode, sampled, second, a, grid, smem, s);
+}
+
+cudaError_t occupancy_stream(int dtype, int mode, bool sampled, bool second, size_t smem, int* nb) {
+  return dtype == 0 ? occupancy_stream_t<float>(mode, sampled, second, smem, nb)
+                    : occupancy_stream_bf16(mode, sampled, second, smem, nb);
 }
 
 __global__ void philox_fill_kernel(uint32_t k0, uint32_t k1, uint32_t c0, uint32_t c1, uint32_t c2,

@@ -1,37 +1,49 @@
-// Streaming kernels of the CM-ASD logits pass (sm_103a).
+// Streaming kernel of the CM-ASD logits pass (sm_103a).
 //
 // Work split.  The present rows (sequence b, drafted position i < k_row[b])
 // are laid end to end into one stream of rows * V logits per tensor, and the
-// launched warps (a persistent grid: every SM filled to its occupancy) each
-// take an equal contiguous slice of that stream.  A slice crosses at most a
-// few row boundaries; each piece of a row it covers is a "segment".
+// launched warps (a persistent grid: one 768-thread CTA per SM) each take one
+// contiguous slice of that stream: whole-warp pieces of one row when there are
+// at least as many warps as rows, equal runs of 16-byte vectors otherwise.
+// Each piece of a row inside a slice is a "segment".
 //
-// Memory pipeline.  Each warp owns a ring of kStages shared-memory stages; a
-// stage holds a 1 KB chunk of the drafter row and the matching 1 KB of the
-// target row, filled by bulk copies (cp.async.bulk, TMA) that complete on the
-// stage's mbarrier.  Lane 0 keeps kStages chunks in flight ahead of the warp,
-// across segment boundaries; the warp reads each landed chunk with 128-bit
-// shared loads.  The unaligned head and tail of a segment (fewer than 16
-// bytes each) are read directly from global memory.
+// Memory pipeline.  A lane's 16-byte vectors in a segment are those with index
+// lane + 32 t; it reads CMSD_UNROLL of each tensor per stage with streaming
+// loads (ld.global.nc, no L1 allocation) into registers, and issues the loads
+// of stage s + 1 before it reduces stage s, so one stage is always in flight.
+// The unaligned head and tail of a segment (under 16 bytes each) are read
+// element by element.
 //
-// Per-element work (online softmax, Sec. III.B(1)): with running maximum m,
-//   s  = sum e^(z - m)
-//   t2 = sum e^(z - m) * (z - m) * log2(e)
-// so that the entropy is H = -sum p log p = ln2 * (log2 s - t2 / s); when m
-// grows to m', s and t2 are rescaled by e^(m - m') (t2 also shifted by
-// s * (m - m') log2 e).  The exponent is evaluated as ex2(z*log2e - m*log2e)
-// with the product m*log2e rounded once and shared by every term of the
-// row, so that rounding cancels in p = e^(z-m)/s.  Pairs of elements go
-// through the packed f32x2 FMA/ADD pipes.  The target row keeps its maximum,
+// Per-element work (online softmax, Sec. III.B(1)): with exponent reference
+// ref (a lane's running maximum, moved only when the maximum exceeds it by
+// kRefSlack), each term is e = 2^(z log2e - ref log2e) and a lane keeps
+//   s  = sum e,   t2 = sum e * (z - ref) log2e
+// so that the entropy is H = -sum p log p = ln2 (log2 s - t2 / s) once s and
+// t2 are shifted to the exact maximum.  A stage first updates the maxima
+// (one reference check per stage), then sums its terms among themselves
+// (pairs of elements through the packed f32x2 FMA/ADD pipes) and adds that
+// stage sum to the lane's sums with compensated (Kahan) addition: after a
+// spike, a lane adds many terms near 1e-6 to a sum near 1, and plain
+// addition would lose most of their bits.  The verifier row keeps its maximum,
 // lowest argmax, the count of logits above the drafted token's (saturating at
-// beta_rank) and, for the sampled rule, its own sum of e^(z - m).
+// beta_rank) and, for the sampled rule, its own sum of exponentials.
 //
-// Reduction.  At the end of a segment the warp merges its lanes with
-// shuffles and writes one Partial.  Per-row and per-sequence arrival
-// counters (atomics, no waiting on other warps) elect the warp that completes
-// a row to merge its partials into the row's results, and the warp that
-// completes a sequence to run the sequence epilogue (first-reject scan, next
-// draft length, output tokens).  Every logit is read from HBM once.
+// Reduction.  At the end of a segment the warp merges its lanes with shuffles
+// and writes one Partial; per-row and per-sequence counters (acquire-release
+// atomics, no waiting) elect the warp that completes a row to merge the row's
+// partials and take its decisions, and the warp that
+// completes a sequence to run the sequence epilogue: first-reject scan, next
+// draft length, output tokens.  For windows of up to 16 positions the
+// sequence counter is one 64-bit word that also carries every position's
+// accept bit and confidence (fixed point), so the epilogue needs no loads.
+//
+// Second pass.  Under the sampled rule the rejected position's token is drawn
+// from the residual max(0, p - q), and with the bonus row the verifier's extra
+// row gives a token when every draft was accepted; both need one more pass
+// over one row of the sequence after its epilogue.  The epilogue queues a
+// record for each sequence that needs one; the resample kernel, launched as a
+// programmatic dependent of this one, splits the queued rows' groups evenly
+// over its warps.  Every logit of the pass proper is read once.
 //
 // -inf logits (masked vocabulary) are clamped to -2^100 before the drafter
 // arithmetic so that e^(z-m) * (z-m) is 0, not NaN.
@@ -57,6 +69,8 @@ template <> struct Elem<uint16_t> {
   }
 };
 
+constexpr int kFixedShift = 36;          // confidence in the sequence word: C * 2^36
+
 // ---------------------------------------------------------------------------
 // per-lane running state
 // ---------------------------------------------------------------------------
@@ -64,26 +78,20 @@ template <> struct Elem<uint16_t> {
 // Each lane walks its elements in increasing index order and keeps, without
 // branches: the exact running maximum and the first vector (or single
 // element) in which it was reached; the exact index inside that vector is
-// resolved at the end of the segment by the lane(s) holding the segment
-// maximum, so the lowest index among equal maxima survives.  The exponent
-// reference `ref` of the sums moves only when the maximum has grown more
-// than kRefSlack above it (rare), so every term is e^(z - ref) <= e^kRefSlack
-// and the final shift to the exact maximum loses no precision.
+// resolved at the end of the segment, so the lowest index among equal maxima
+// survives.  The exponent reference `ref` of the sums moves only when the
+// maximum has grown more than kRefSlack above it (rare), so every term is
+// e^(z - ref) <= e^kRefSlack and the final shift to the exact maximum loses
+// no precision.
 
 constexpr float kRefSlack = 4.0f;   // nats
 
-#ifndef CMSD_DRAFT_PACKED
-#define CMSD_DRAFT_PACKED 1
-#endif
-#ifndef CMSD_TARGET_PACKED
-#define CMSD_TARGET_PACKED 1
-#endif
-
 struct DLane {               // drafter
-  float m;                   // exact running max (of clamped logits)
+  float m;                   // exact running max of the raw logits (kNegInit: none yet)
   float ref;                 // exponent reference of s and t
   u64 negrL;                 // -(ref*log2e) in both halves
-  u64 s, t;                  // packed (even, odd) sums of e and of e*x, relative to ref
+  float s, cs;               // sum of e, and its compensation (Kahan)
+  float t, ct;               // sum of e*x, and its compensation
   float f1, f2;              // top-2 of elements taken one at a time (all f32 data)
   uint32_t T1, T2;           // top-2 of bf16 vector elements, per half-word lane
   int pos, posw;             // first unit (start, width) that reached m
@@ -93,7 +101,7 @@ struct TLane {               // target
   float M;                   // exact running max
   float ref;
   u64 negrL;
-  u64 s;                     // packed partial sums of e^(z - ref)
+  float s, cs;               // sum of e^(z - ref), and its compensation
   float thr;                 // PAPER rule: elements above thr may be counted
   int pos, posw;
   int cnt;
@@ -103,7 +111,7 @@ __device__ __forceinline__ void dlane_init(DLane& d) {
   d.m = kNegInit;
   d.ref = kNegInit;
   d.negrL = dup2(-mlog2e(kNegInit));
-  d.s = d.t = 0ull;
+  d.s = d.cs = d.t = d.ct = 0.f;
   d.f1 = d.f2 = kNegInit;
   d.T1 = d.T2 = kNegInf2;
   d.pos = kIntMax;
@@ -113,7 +121,7 @@ __device__ __forceinline__ void tlane_init(TLane& t, float c, int beta) {
   t.M = kNegInit;
   t.ref = kNegInit;
   t.negrL = dup2(-mlog2e(kNegInit));
-  t.s = 0ull;
+  t.s = t.cs = 0.f;
   t.pos = kIntMax;
   t.posw = 0;
   t.cnt = 0;
@@ -121,63 +129,56 @@ __device__ __forceinline__ void tlane_init(TLane& t, float c, int beta) {
   if (beta > 0) t.thr = c;   // c is a pending load: read it only when needed
 }
 
+// Compensated (Kahan) accumulation s += x; the sum is s - c.
+__device__ __forceinline__ void kahan(float& s, float& c, float x) {
+  const float y = __fsub_rn(x, c);
+  const float u = __fadd_rn(s, y);
+  c = __fsub_rn(__fsub_rn(u, s), y);
+  s = u;
+}
+
+// The drafter's maximum as the exponent arithmetic sees it: masked (-inf)
+// logits count as -2^100.
+__device__ __forceinline__ float d_mexp(const DLane& d) { return fmaxf(d.m, neg_clamp()); }
+
 // move the exponent reference up to mx: s *= e^(ref - mx), t likewise
-// (shifted by s * (ref - mx) log2e)
+// (shifted by s * (ref - mx) log2e); the compensations are folded in
 __device__ __forceinline__ void d_reref(DLane& d, float mx) {
   const float nrL = mlog2e(mx);
   const float dd = __fsub_rn(-lo32f(d.negrL), nrL);    // (ref_old - ref_new) log2e <= 0
-  const u64 sc = dup2(ex2(dd));
-  d.t = mul2(sc, fma2(d.s, dup2(dd), d.t));
-  d.s = mul2(d.s, sc);
+  const float sc = ex2(dd);
+  const float s0 = __fsub_rn(d.s, d.cs), t0 = __fsub_rn(d.t, d.ct);
+  d.t = sc * fmaf(s0, dd, t0);
+  d.s = s0 * sc;
+  d.cs = d.ct = 0.f;
   d.ref = mx;
   d.negrL = dup2(-nrL);
 }
 __device__ __forceinline__ void t_reref(TLane& t, float mx) {
   const float nrL = mlog2e(mx);
-  t.s = mul2(t.s, dup2(ex2(__fsub_rn(-lo32f(t.negrL), nrL))));
+  t.s = __fsub_rn(t.s, t.cs) * ex2(__fsub_rn(-lo32f(t.negrL), nrL));
+  t.cs = 0.f;
   t.ref = mx;
   t.negrL = dup2(-nrL);
 }
 
-// accumulate a pair of (clamped) drafter logits given as packed floats
-__device__ __forceinline__ void d_acc(DLane& d, u64 z) {
-#if CMSD_DRAFT_PACKED
-  const u64 x = fma2(z, dup2(kLog2e), d.negrL);
-  const u64 e = ex2_2(x);
-  d.s = add2(d.s, e);
-  d.t = fma2(e, x, d.t);
-#else
-  const float nr = lo32f(d.negrL);
-  const float xa = fmaf(lo32f(z), kLog2e, nr), xb = fmaf(hi32f(z), kLog2e, nr);
-  const float ea = ex2(xa), eb = ex2(xb);
-  d.s = pack2(lo32f(d.s) + ea, hi32f(d.s) + eb);
-  d.t = pack2(fmaf(ea, xa, lo32f(d.t)), fmaf(eb, xb, hi32f(d.t)));
-#endif
-}
-__device__ __forceinline__ void t_acc(TLane& t, u64 z) {
-#if CMSD_TARGET_PACKED
-  t.s = add2(t.s, ex2_2(fma2(z, dup2(kLog2e), t.negrL)));
-#else
-  const float nr = lo32f(t.negrL);
-  t.s = pack2(lo32f(t.s) + ex2(fmaf(lo32f(z), kLog2e, nr)), hi32f(t.s) + ex2(fmaf(hi32f(z), kLog2e, nr)));
-#endif
-}
-
 // --- drafter: one element at a time (segment heads/tails) --------------------
 __device__ __forceinline__ void d_scalar(DLane& d, float z, int v) {
-  z = fmaxf(z, neg_clamp());
   d.f2 = fmaxf(d.f2, fminf(d.f1, z));
   d.f1 = fmaxf(d.f1, z);
   if (z > d.m) { d.pos = v; d.posw = 1; }
   d.m = fmaxf(d.m, z);
-  if (z > d.ref + kRefSlack) d_reref(d, z);
-  d_acc(d, pack2(z, kNegInit));          // the second half adds e = 0
+  const float me = d_mexp(d);
+  if (me > d.ref + kRefSlack) d_reref(d, me);
+  const float x = fmaf(fmaxf(z, neg_clamp()), kLog2e, lo32f(d.negrL));
+  const float e = ex2(x);
+  kahan(d.s, d.cs, e);
+  kahan(d.t, d.ct, e * x);
 }
 
-// --- drafter: 8 bf16 ---------------------------------------------------------
-__device__ __forceinline__ void d_vec(DLane& d, uint4 q, int v) {
-  const uint32_t w[4] = {bmax2(q.x, kNegClamp2), bmax2(q.y, kNegClamp2), bmax2(q.z, kNegClamp2),
-                         bmax2(q.w, kNegClamp2)};
+// --- drafter, maximum phase: top-2 and the first vector of the maximum --------
+__device__ __forceinline__ void d_vmax(DLane& d, uint4 q, int v) {
+  const uint32_t w[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     d.T2 = bmax2(d.T2, bmin2(d.T1, w[k]));
@@ -188,15 +189,9 @@ __device__ __forceinline__ void d_vec(DLane& d, uint4 q, int v) {
   d.pos = up ? v : d.pos;
   d.posw = up ? 8 : d.posw;
   d.m = fmaxf(d.m, mx);
-  if (mx > d.ref + kRefSlack) d_reref(d, mx);
-#pragma unroll
-  for (int k = 0; k < 4; ++k) d_acc(d, bf2_to_f2(w[k]));
 }
-
-// --- drafter: 4 f32 ------------------------------------------------------------
-__device__ __forceinline__ void d_vec(DLane& d, float4 q, int v) {
-  const float nc = neg_clamp();
-  const float z[4] = {fmaxf(q.x, nc), fmaxf(q.y, nc), fmaxf(q.z, nc), fmaxf(q.w, nc)};
+__device__ __forceinline__ void d_vmax(DLane& d, float4 q, int v) {
+  const float z[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     d.f2 = fmaxf(d.f2, fminf(d.f1, z[k]));
@@ -206,9 +201,27 @@ __device__ __forceinline__ void d_vec(DLane& d, float4 q, int v) {
   d.pos = up ? v : d.pos;
   d.posw = up ? 4 : d.posw;
   d.m = fmaxf(d.m, d.f1);
-  if (d.f1 > d.ref + kRefSlack) d_reref(d, d.f1);
-  d_acc(d, pack2(z[0], z[1]));
-  d_acc(d, pack2(z[2], z[3]));
+}
+
+// --- drafter, exponent phase: the vector's terms, summed among themselves ----
+__device__ __forceinline__ void d_vexp(const DLane& d, uint4 q, u64& ss, u64& ts) {
+  const uint32_t w[4] = {bmax2(q.x, kNegClamp2), bmax2(q.y, kNegClamp2), bmax2(q.z, kNegClamp2),
+                         bmax2(q.w, kNegClamp2)};
+  const u64 L = dup2(kLog2e);
+  const u64 x0 = fma2(bf2_to_f2(w[0]), L, d.negrL), x1 = fma2(bf2_to_f2(w[1]), L, d.negrL);
+  const u64 x2 = fma2(bf2_to_f2(w[2]), L, d.negrL), x3 = fma2(bf2_to_f2(w[3]), L, d.negrL);
+  const u64 e0 = ex2_2(x0), e1 = ex2_2(x1), e2 = ex2_2(x2), e3 = ex2_2(x3);
+  ss = add2(ss, add2(add2(e0, e1), add2(e2, e3)));
+  ts = add2(ts, fma2(e3, x3, fma2(e2, x2, fma2(e1, x1, mul2(e0, x0)))));
+}
+__device__ __forceinline__ void d_vexp(const DLane& d, float4 q, u64& ss, u64& ts) {
+  const float nc = neg_clamp();
+  const u64 L = dup2(kLog2e);
+  const u64 x0 = fma2(pack2(fmaxf(q.x, nc), fmaxf(q.y, nc)), L, d.negrL);
+  const u64 x1 = fma2(pack2(fmaxf(q.z, nc), fmaxf(q.w, nc)), L, d.negrL);
+  const u64 e0 = ex2_2(x0), e1 = ex2_2(x1);
+  ss = add2(ss, add2(e0, e1));
+  ts = add2(ts, fma2(e1, x1, mul2(e0, x0)));
 }
 
 // --- target -----------------------------------------------------------------------
@@ -218,13 +231,12 @@ __device__ __forceinline__ void t_scalar(TLane& t, float z, int v, float c, int 
   t.M = fmaxf(t.M, z);
   if (t.cnt < beta && z > c) ++t.cnt;
   if (SAMPLED) {
-    if (z > t.ref + kRefSlack) t_reref(t, z);
-    t_acc(t, pack2(z, -pos_inf()));
+    if (t.M > t.ref + kRefSlack) t_reref(t, t.M);
+    kahan(t.s, t.cs, ex2(fmaf(z, kLog2e, lo32f(t.negrL))));
   }
 }
 
-template <bool SAMPLED>
-__device__ __forceinline__ void t_vec(TLane& t, uint4 q, int v, float c, int beta) {
+__device__ __forceinline__ void t_vmax(TLane& t, uint4 q, int v, float c, int beta) {
   const uint32_t w[4] = {q.x, q.y, q.z, q.w};
   const uint32_t a = bmax2(bmax2(w[0], w[1]), bmax2(w[2], w[3]));
   const float vmax = fmaxf(bf_lo(a), bf_hi(a));
@@ -237,15 +249,8 @@ __device__ __forceinline__ void t_vec(TLane& t, uint4 q, int v, float c, int bet
     for (int k = 0; k < 4; ++k) t.cnt += (bf_lo(w[k]) > c) + (bf_hi(w[k]) > c);
     if (t.cnt >= beta) t.thr = pos_inf();
   }
-  if (SAMPLED) {
-    if (vmax > t.ref + kRefSlack) t_reref(t, vmax);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) t_acc(t, bf2_to_f2(w[k]));
-  }
 }
-
-template <bool SAMPLED>
-__device__ __forceinline__ void t_vec(TLane& t, float4 q, int v, float c, int beta) {
+__device__ __forceinline__ void t_vmax(TLane& t, float4 q, int v, float c, int beta) {
   const float z[4] = {q.x, q.y, q.z, q.w};
   const float vmax = fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3]));
   const bool up = vmax > t.M;
@@ -256,23 +261,31 @@ __device__ __forceinline__ void t_vec(TLane& t, float4 q, int v, float c, int be
     t.cnt += (z[0] > c) + (z[1] > c) + (z[2] > c) + (z[3] > c);
     if (t.cnt >= beta) t.thr = pos_inf();
   }
-  if (SAMPLED) {
-    if (vmax > t.ref + kRefSlack) t_reref(t, vmax);
-    t_acc(t, pack2(z[0], z[1]));
-    t_acc(t, pack2(z[2], z[3]));
-  }
 }
 
-// s and t of a drafter lane relative to its exact maximum m
+__device__ __forceinline__ void t_vexp(const TLane& t, uint4 q, u64& ss) {
+  const u64 L = dup2(kLog2e);
+  const u64 e0 = ex2_2(fma2(bf2_to_f2(q.x), L, t.negrL)), e1 = ex2_2(fma2(bf2_to_f2(q.y), L, t.negrL));
+  const u64 e2 = ex2_2(fma2(bf2_to_f2(q.z), L, t.negrL)), e3 = ex2_2(fma2(bf2_to_f2(q.w), L, t.negrL));
+  ss = add2(ss, add2(add2(e0, e1), add2(e2, e3)));
+}
+__device__ __forceinline__ void t_vexp(const TLane& t, float4 q, u64& ss) {
+  const u64 L = dup2(kLog2e);
+  const u64 e0 = ex2_2(fma2(pack2(q.x, q.y), L, t.negrL));
+  const u64 e1 = ex2_2(fma2(pack2(q.z, q.w), L, t.negrL));
+  ss = add2(ss, add2(e0, e1));
+}
+
+// s and t of a drafter lane relative to its maximum (as the exponents see it)
 __device__ __forceinline__ void d_final(const DLane& d, float& s, float& t2) {
-  const float dd = __fsub_rn(-lo32f(d.negrL), mlog2e(d.m));   // (ref - m) log2e <= 0
+  const float dd = __fsub_rn(-lo32f(d.negrL), mlog2e(d_mexp(d)));   // (ref - m) log2e <= 0
   const float sc = ex2(dd);
-  const float s0 = lo32f(d.s) + hi32f(d.s);
+  const float s0 = __fsub_rn(d.s, d.cs);
   s = s0 * sc;
-  t2 = sc * fmaf(s0, dd, lo32f(d.t) + hi32f(d.t));
+  t2 = sc * fmaf(s0, dd, __fsub_rn(d.t, d.ct));
 }
 __device__ __forceinline__ float t_final(const TLane& t) {
-  return (lo32f(t.s) + hi32f(t.s)) * ex2(__fsub_rn(-lo32f(t.negrL), mlog2e(t.M)));
+  return __fsub_rn(t.s, t.cs) * ex2(__fsub_rn(-lo32f(t.negrL), mlog2e(t.M)));
 }
 
 template <typename T> struct VecT;
@@ -296,10 +309,8 @@ __device__ __forceinline__ float logit_at(uint4 q, int k) {
   return __uint_as_float(w);
 }
 
-// First index in the unit (start pos, width w) whose value equals m (drafter
-// values clamped as in the streaming pass when `clamp`).  A unit of width > 1
-// is one aligned 16-byte vector of the row: it is read with a single load
-// and searched in registers.
+// First index in a 16-byte vector whose value equals m (drafter values
+// clamped as in the streaming pass when `clamp`).
 template <typename T>
 __device__ __forceinline__ int first_in_vec(uint4 q, float m, bool clamp) {
   const float nc = neg_clamp();
@@ -311,11 +322,6 @@ __device__ __forceinline__ int first_in_vec(uint4 q, float m, bool clamp) {
     k = (z == m) ? j : k;
   }
   return k;
-}
-template <typename T>
-__device__ __forceinline__ int first_equal(const T* row, int pos, int w, float m, bool clamp) {
-  if (w <= 1) return pos;
-  return pos + first_in_vec<T>(__ldcg(reinterpret_cast<const uint4*>(row + pos)), m, clamp);
 }
 
 // ---------------------------------------------------------------------------
@@ -415,12 +421,6 @@ __device__ __forceinline__ void fold_t(TRed& a, const TRed& b) {
 // work split
 // ---------------------------------------------------------------------------
 
-__device__ __forceinline__ int eff_warps(int64_t N, int64_t min_len, int nwarps) {
-  int64_t w = N / min_len;
-  if (w < 1) w = 1;
-  if (w > nwarps) w = nwarps;
-  return (int)w;
-}
 __device__ __forceinline__ int64_t stream_min_len(int V) {
   const int64_t a = (int64_t)V / 64 + 64;
   return a > 2048 ? a : 2048;
@@ -533,6 +533,8 @@ __device__ __forceinline__ void map_row(const StreamArgs& a, const int* pref, in
 
 // Geometry of one segment: row elements [v0, v1), with the 16-byte aligned
 // body [va, vb) (a whole number of vectors) between a head and a tail.
+// r = b*K + i indexes positions (drafter rows, tokens, per-position outputs);
+// the verifier row of the position is b*Kt + i.
 struct Seg {
   int ar, b, i, r;
   int v0, v1, va, vb;
@@ -540,7 +542,7 @@ struct Seg {
 
 template <typename T>
 __device__ __forceinline__ Seg make_seg(const StreamArgs& a, const int* pref, int64_t e, int64_t e_end,
-                                        const void* base) {
+                                        const void* base, bool base_is_target) {
   constexpr int VEC = Elem<T>::kVec;
   Seg s;
   s.ar = (int)(e / a.V);
@@ -549,7 +551,8 @@ __device__ __forceinline__ Seg make_seg(const StreamArgs& a, const int* pref, in
   s.v1 = s.v0 + len;
   map_row(a, pref, s.ar, s.b, s.i);
   s.r = s.b * a.K + s.i;
-  const uintptr_t addr = (uintptr_t)((const T*)base + (size_t)s.r * (size_t)a.V + s.v0);
+  const size_t row = base_is_target ? (size_t)s.b * a.Kt + s.i : (size_t)s.r;
+  const uintptr_t addr = (uintptr_t)((const T*)base + row * (size_t)a.V + s.v0);
   const int mis = (int)((addr & 15) / sizeof(T));
   const int head = mis ? min(VEC - mis, len) : 0;
   s.va = s.v0 + head;
@@ -561,77 +564,91 @@ __device__ __forceinline__ Seg make_seg(const StreamArgs& a, const int* pref, in
 // sequence epilogue: first-reject scan, next draft length, output tokens
 // ---------------------------------------------------------------------------
 
+// Sec. III.B(b): k = min(k_max, max(k_min, floor(alpha * Cbar * k_max))), with
+// Cbar = csum 2^-36 / kb from the window's confidences in fixed point: with
+// alpha = ma 2^ea, floor(alpha csum 2^-36 k_max / kb) is formed exactly in
+// integer arithmetic.  A constant k when k_fixed > 0 (the fixed-k variants of
+// the ablation, Table III).
+__device__ __forceinline__ int next_k(const StreamArgs& a, unsigned long long csum, int kb) {
+  if (a.k_fixed > 0) return a.k_fixed;
+  if (kb <= 0) return a.k_min;
+  const uint32_t bits = __float_as_uint(a.alpha);                    // 0 < alpha <= 1, normal
+  const int ea = (int)((bits >> 23) & 0xFFu) - 150;                  // alpha = ma 2^ea, ea <= -23
+  const unsigned long long t = (unsigned long long)((bits & 0x7FFFFFu) | 0x800000u) *
+                               (unsigned long long)a.k_max;           // < 2^35
+  const unsigned long long lo = t * csum, hi = __umul64hi(t, csum);
+  const int sh = kFixedShift - ea;                                    // >= 59
+  const unsigned long long q = sh >= 128 ? 0ull
+                             : sh >= 64 ? (hi >> (sh - 64))
+                                        : ((lo >> sh) | (hi << (64 - sh)));
+  const unsigned long long kk = q / (unsigned long long)kb;
+  const int k = kk > (unsigned long long)a.k_max ? a.k_max : (int)kk;
+  return k < a.k_min ? a.k_min : k;
+}
+
+// Queue the sequence's second-pass record, if it needs one.
+__device__ __forceinline__ void publish(const StreamArgs& a, int b, int kind, int pos) {
+  if (kind == kSeqNone) return;
+  const int slot = atomicAdd(a.ws.rec_count, 1);
+  if (slot < a.B) a.ws.rec[slot] = make_int4(b, pos, kind, 0);
+}
+
 template <int MODE, bool SAMPLED>
-__device__ void seq_epilogue(const StreamArgs& a, int b, int kb, int lane) {
+__device__ __forceinline__ int seq_kind(const StreamArgs& a, int n, int kb) {
+  if (SAMPLED && n < kb) return kSeqResidual;
+  if (a.bonus && n == kb) return kSeqBonus;
+  return kSeqNone;
+}
+
+// One position per lane; write the outputs of sequence b given n, the accept
+// bits and the drafted tokens (tok: this lane's position's token).
+//   out_tokens: accepted drafts, then at n the correction (PAPER rule: already
+//   written by the row merge of position n; sampled rule: -1 until the second
+//   pass writes it), -1 after; with the bonus row, slot k_b holds -1 until the
+//   second pass writes the verifier's token.
+template <int MODE, bool SAMPLED>
+__device__ __forceinline__ void write_outputs(const StreamArgs& a, int b, int kb, int n, int i, int tok,
+                                              bool acc_i) {
+  if (i < a.Ko) {
+    const bool mine = (i == n && n < kb && !SAMPLED);
+    if (!mine) a.out_tokens[(size_t)b * a.Ko + i] = (i < n) ? tok : -1;
+  }
+  if (a.accept && i < a.K) a.accept[(size_t)b * a.K + i] = (i < kb && acc_i) ? 1 : 0;
+}
+
+// Epilogue of a window of at most 16 positions: everything comes in the
+// sequence word (rows merged | accept bits << 6 | sum of C * 2^36 << 22);
+// tok is this lane's prefetched drafted token.
+template <int MODE, bool SAMPLED, bool PH2>
+__device__ __forceinline__ void seq_epilogue_packed(const StreamArgs& a, int b, int kb, unsigned long long word, int tok,
+                                    int lane) {
+  const unsigned bits = (unsigned)(word >> 6) & 0xFFFFu;
+  const unsigned rej = ~bits & ((1u << kb) - 1u);
+  const int n = rej ? __ffs(rej) - 1 : kb;
+  if (lane == 0) {
+    if (MODE != kModeVerify && a.k_next) a.k_next[b] = next_k(a, word >> 22, kb);
+    if (MODE != kModeConf) a.n_accept[b] = n;
+    a.ws.seq_word[b] = 0ull;
+  }
+  if (MODE != kModeConf) {
+    write_outputs<MODE, SAMPLED>(a, b, kb, n, lane, tok, (bits >> lane) & 1u);
+    if (PH2 && lane == 0) publish(a, b, seq_kind<MODE, SAMPLED>(a, n, kb), n);
+  }
+}
+
+// Epilogue of a longer window: reads the accept bits and confidences of the
+// window's positions from the workspace.
+template <int MODE, bool SAMPLED, bool PH2>
+__device__ __forceinline__ void seq_epilogue_loads(const StreamArgs& a, int b, int kb, int lane) {
   const Workspace& W = a.ws;
   const int base = b * a.K;
-  if (a.K <= 32) {
-    // one position per lane: every value the outputs need is requested at once
-    const int i = lane;
-    const bool valid = i < kb;
-    int acc = 1, tok = -1, tmx = 0;
-    float cf = 0.f;
-    float2 ts = make_float2(0.f, 1.f), ds = make_float2(0.f, 1.f);
-    if (valid) {
-      if (MODE != kModeConf) {
-        acc = __ldcg(W.row_acc + base + i);
-        tok = __ldg(a.tokens + base + i);
-        tmx = __ldcg(W.row_targmax + base + i);
-        if (SAMPLED) {
-          ts = __ldcg(W.row_tstat + base + i);
-          ds = __ldcg(W.row_dstat + base + i);
-        }
-      }
-      if (MODE != kModeVerify) cf = __ldcg(W.row_conf + base + i);
-    }
-    const unsigned rej = __ballot_sync(kFull, valid && !acc);
-    const int n = rej ? __ffs(rej) - 1 : kb;
-    if (MODE != kModeVerify) {
-      const float csum = warp_sum_f(cf);
-      if (lane == 0 && a.k_next) {
-        int k = a.k_min;
-        if (kb > 0) {
-          const float cbar = csum / (float)kb;
-          const float x = a.alpha * cbar * (float)a.k_max;
-          k = (int)floorf(x);
-          k = k < a.k_min ? a.k_min : (k > a.k_max ? a.k_max : k);
-        }
-        a.k_next[b] = k;
-      }
-    }
-    if (MODE != kModeConf) {
-      if (i < a.K) {
-        int ot = -1;
-        if (i < n) ot = tok;
-        else if (i == n && n < kb) ot = SAMPLED ? -1 : tmx;
-        a.out_tokens[base + i] = ot;
-        if (a.accept) a.accept[base + i] = valid ? (unsigned char)(acc != 0) : 0;
-      }
-      if (lane == 0) a.n_accept[b] = n;
-      if (SAMPLED && i == n && n < kb) {
-        const int slot = atomicAdd(W.rej_count, 1);
-        if (slot < a.B) {
-          RejRec q;
-          q.r = base + n; q.b = b; q.n = n;
-          q.targmax = tmx;
-          q.MLt = ts.x; q.invSt = 1.0f / ts.y;
-          q.MLd = ds.x; q.invSd = 1.0f / ds.y;
-          W.rej[slot] = q;
-        } else {
-          atomicOr(W.err, 4u);   // queue not drained by a previous call: workspace misuse
-        }
-      }
-    }
-    if (lane == 0) W.seq_done[b] = 0;
-    return;
-  }
   int n = kb;
-  float csum = 0.f;
+  unsigned long long csum = 0ull;
   for (int i0 = 0; i0 < kb; i0 += 32) {
     const int i = i0 + lane;
     const bool valid = i < kb;
     int acc = 1;
-    float cf = 0.f;
+    unsigned long long cf = 0ull;
     if (valid) {
       if (MODE != kModeConf) acc = __ldcg(W.row_acc + base + i);
       if (MODE != kModeVerify) cf = __ldcg(W.row_conf + base + i);
@@ -641,142 +658,176 @@ __device__ void seq_epilogue(const StreamArgs& a, int b, int kb, int lane) {
     csum += cf;
   }
   if (MODE != kModeVerify) {
-    csum = warp_sum_f(csum);
-    if (lane == 0 && a.k_next) {
-      int k = a.k_min;
-      if (kb > 0) {
-        const float cbar = csum / (float)kb;
-        const float x = a.alpha * cbar * (float)a.k_max;
-        k = (int)floorf(x);
-        k = k < a.k_min ? a.k_min : (k > a.k_max ? a.k_max : k);
-      }
-      a.k_next[b] = k;
-    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) csum += __shfl_xor_sync(kFull, csum, o);
+    if (lane == 0 && a.k_next) a.k_next[b] = next_k(a, csum, kb);
   }
   if (MODE != kModeConf) {
-    for (int i = lane; i < a.K; i += 32) {
-      int tok = -1;
-      if (i < n) {
-        tok = __ldg(a.tokens + base + i);
-      } else if (i == n && n < kb) {
-        tok = SAMPLED ? -1 : __ldcg(W.row_targmax + base + n);
-      }
-      a.out_tokens[base + i] = tok;
-      if (a.accept) a.accept[base + i] = (i < kb) ? (unsigned char)(__ldcg(W.row_acc + base + i) != 0) : 0;
+    for (int i = lane; i < a.Ko; i += 32) {
+      const int tok = (i < n) ? __ldg(a.tokens + base + i) : -1;
+      const bool acc_i = (i < kb) ? (__ldcg(W.row_acc + base + i) != 0) : false;
+      write_outputs<MODE, SAMPLED>(a, b, kb, n, i, tok, acc_i);
     }
-    if (lane == 0) {
-      a.n_accept[b] = n;
-      if (SAMPLED && n < kb) {
-        const int slot = atomicAdd(W.rej_count, 1);
-        if (slot < a.B) {
-          const int r = base + n;
-          const float2 ts = __ldcg(W.row_tstat + r);
-          const float2 ds = __ldcg(W.row_dstat + r);
-          RejRec q;
-          q.r = r; q.b = b; q.n = n;
-          q.targmax = __ldcg(W.row_targmax + r);
-          q.MLt = ts.x; q.invSt = 1.0f / ts.y;
-          q.MLd = ds.x; q.invSd = 1.0f / ds.y;
-          W.rej[slot] = q;
-        } else {
-          atomicOr(W.err, 4u);   // queue not drained by a previous call: workspace misuse
-        }
-      }
-    }
+    if (lane == 0) a.n_accept[b] = n;
   }
   if (lane == 0) W.seq_done[b] = 0;
-}
-
-
-// ---------------------------------------------------------------------------
-// row results from the merged statistics
-// ---------------------------------------------------------------------------
-
-template <typename T, int MODE, bool SAMPLED>
-__device__ void row_results(const StreamArgs& a, int r, int b, int i, const DRed& d, const TRed& t,
-                            float c_tgt, float zd) {
-  const Workspace& W = a.ws;
-  float C = 0.f, MLd = 0.f, Sd = 1.f;
-  if (MODE != kModeVerify) {
-    MLd = mlog2e(d.m);
-    Sd = d.s;
-    const float H = kLn2 * (log2f(d.s) - d.t2 / d.s);
-    const float margin = (d.top2 <= neg_clamp()) ? pos_inf() : d.m - d.top2;
-    const float psm = (1.0f - exp2f(fmaf(d.top2, kLog2e, -MLd))) / d.s;
-    const float Vf = (float)a.V;
-    const float c_ent = 1.0f - H / logf(Vf);
-    const float c_mar = 1.0f / (1.0f + expf(-a.beta_sig * margin));
-    const float c_soft = psm / (1.0f - 1.0f / Vf);
-    C = a.lam0 * c_ent + a.lam1 * c_mar + a.lam2 * c_soft;
-    C = fminf(1.0f, fmaxf(0.0f, C));
-    if (a.H) a.H[r] = H;
-    if (a.margin) a.margin[r] = margin;
-    if (a.argmax) a.argmax[r] = d.idx;
-    if (a.conf) a.conf[r] = C;
-    if (a.lse) a.lse[r] = d.m + kLn2 * log2f(d.s);
-  } else {
-    C = __ldg(a.conf_in + r);
-  }
-  W.row_conf[r] = C;
-  if (MODE != kModeConf) {
-    const float tau = (a.tau_sign >= 0) ? a.tau_base + a.gamma * (1.0f - C)
-                                        : a.tau_base + a.gamma * C;
-    const bool rank_ok = a.beta_rank <= 0 || t.cnt < a.beta_rank;
-    bool acc;
-    const float MLt = mlog2e(t.m);
-    if (!SAMPLED) {
-      const float gap = t.m - c_tgt;
-      acc = rank_ok && gap <= tau;
-    } else {
-      const float p = exp2f(fmaf(c_tgt, kLog2e, -MLt)) / t.s;
-      float q;
-      if (MODE == kModeFused) {
-        q = exp2f(fmaf(zd, kLog2e, -MLd)) / Sd;
-      } else {
-        const float lse = __ldg(a.lse_in + r);
-        q = expf(zd - lse);
-        MLd = lse * kLog2e;
-        Sd = 1.0f;
-      }
-      const U4 w = philox4x32_10(U4{0u, (uint32_t)b, (uint32_t)i, iter_word(a.iteration, kPurposeAccept)},
-                                 seed_lo(a.seed), seed_hi(a.seed));
-      const float u = word_to_unit(w.x);
-      acc = rank_ok && (u * q < expf(tau) * p);
-      W.row_dstat[r] = make_float2(MLd, Sd);
-      W.row_tstat[r] = make_float2(MLt, t.s);
-    }
-    W.row_acc[r] = acc ? 1 : 0;
-    W.row_targmax[r] = t.idx;
-  }
+  if (MODE != kModeConf && PH2 && lane == 0) publish(a, b, seq_kind<MODE, SAMPLED>(a, n, kb), n);
 }
 
 // ---------------------------------------------------------------------------
-// the streaming kernel
+// row results from the merged statistics (lane 0 of the merging warp)
 // ---------------------------------------------------------------------------
 //
-// Every warp owns one contiguous slice of the stream.  Within each segment
-// (the part of one row inside the slice) a lane's 16-byte vectors are those
-// with index lane + 32 t, CMSD_UNROLL of each tensor per stage; the loads of
-// stage s+1 are issued into registers before stage s is reduced, so every
-// lane keeps one stage in flight and no lane waits on another.  A segment's
-// unaligned head and tail (under 16 bytes each) are read directly.
-// At the end of a segment the warp reduces its lanes and writes one Partial;
-// the warp that completes a row merges the row and, when it completes a
-// sequence, runs the sequence epilogue.  Warps never wait on each other.
+// All in fp32 (fp64 issues slowly on this part), arranged so that no step
+// loses more than a rounding: exponentials take arguments that are exact
+// differences of logits, the sums' scale 2^(m log2e - fl(m log2e)) is the
+// exact rounding residual of one product, log2 s is split into the exponent
+// of s and the log2 of its mantissa, and the confidence is summed with
+// error-free transformations into fixed point (C * 2^36).
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+// log2 s = e + log2(mantissa), mantissa in [1, 2)
+__device__ __forceinline__ float log2_split(float s) {
+  int e;
+  const float m = frexpf(s, &e);      // s = m 2^e, m in [0.5, 1)
+  return (float)(e - 1) + log2f(2.0f * m);
 }
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+// 2^(a - b) for floats a, b with a - b in the normal range: the difference
+// is formed exactly as hi + lo (TwoSum), then 2^n ex2(hi - n + lo)
+__device__ __forceinline__ float exp2_diff(float a, float b) {
+  const float nb = -b;
+  const float hi = __fadd_rn(a, nb);
+  const float z = __fsub_rn(hi, a);
+  const float lo = __fadd_rn(__fsub_rn(a, __fsub_rn(hi, z)), __fsub_rn(nb, z));
+  const float n = rintf(hi);
+  return ldexpf(exp2f(__fadd_rn(__fsub_rn(hi, n), lo)), (int)n);
+}
 
-#ifndef CMSD_MIN_BLOCKS
-#define CMSD_MIN_BLOCKS 1
-#endif
+// lambda . c as an unevaluated sum hi + lo (error-free products and sums)
+__device__ __forceinline__ void dot3_exact(float l0, float c0, float l1, float c1, float l2, float c2,
+                                           float& hi, float& lo) {
+  const float p0 = __fmul_rn(l0, c0), p1 = __fmul_rn(l1, c1), p2 = __fmul_rn(l2, c2);
+  float err = fmaf(l0, c0, -p0) + fmaf(l1, c1, -p1) + fmaf(l2, c2, -p2);
+  float s = __fadd_rn(p0, p1);
+  float bb = __fsub_rn(s, p0);
+  err += __fadd_rn(__fsub_rn(p0, __fsub_rn(s, bb)), __fsub_rn(p1, bb));
+  const float s2 = __fadd_rn(s, p2);
+  bb = __fsub_rn(s2, s);
+  err += __fadd_rn(__fsub_rn(s, __fsub_rn(s2, bb)), __fsub_rn(p2, bb));
+  hi = __fadd_rn(s2, err);
+  lo = __fsub_rn(err, __fsub_rn(hi, s2));
+}
+
+constexpr float kFixedScale = 68719476736.0f;   // 2^36
+
+// Called by the whole warp (statistics identical in every lane): the row's
+// exponentials and reciprocals are spread one per lane, so each costs one
+// instruction sequence instead of a chain on one lane.  Lane 0 writes.
+template <typename T, int MODE, bool SAMPLED>
+__device__ __forceinline__ void row_results(const StreamArgs& a, int r, int b, int i, const DRed& d, const TRed& t,
+                                         float c_tgt, float zd, int lane, bool& acc_out,
+                                         unsigned long long& cfx_out) {
+  constexpr bool HAS_D = MODE != kModeVerify;
+  constexpr bool HAS_T = MODE != kModeConf;
+  const Workspace& W = a.ws;
+  const float MLd0 = HAS_D ? mlog2e(d.m) : 0.f;
+  const float MLt = HAS_T ? mlog2e(t.m) : 0.f;
+  const float res_m = HAS_D ? fmaf(d.m, kLog2e, -MLd0) : 0.f;   // exact rounding residuals of m log2e
+  const float res_t = HAS_T ? fmaf(t.m, kLog2e, -MLt) : 0.f;
+  const bool has2 = HAS_D && d.top2 > neg_clamp();
+  const float margin = has2 ? d.m - d.top2 : pos_inf();
+  const float lse_in = (MODE == kModeVerify && SAMPLED) ? __ldg(a.lse_in + r) : 0.f;
+  // one exponential per lane
+  float x = 0.f;
+  if (lane == 0) x = has2 ? d.top2 - d.m : -pos_inf();        // e^(z(2) - m)
+  if (lane == 1) x = -a.beta_sig * margin;                     // sigmoid of the margin
+  if (lane == 2) x = c_tgt - t.m;                              // p, unnormalised
+  if (lane == 3) x = MODE == kModeVerify ? zd - lse_in : zd - d.m;   // q
+  if (lane == 4) x = res_m * kLn2;                             // the sums' scales
+  if (lane == 5) x = res_t * kLn2;
+  const float ex = expf(x);
+  const float e_mar = __shfl_sync(kFull, ex, 1);
+  // one reciprocal per lane
+  float den = 1.f;
+  if (lane == 0 && HAS_D) den = d.s;
+  if (lane == 1) den = 1.0f + e_mar;
+  if (lane == 2 && HAS_T) den = t.s;
+  const float rc = 1.0f / den;
+  const float inv_s = __shfl_sync(kFull, rc, 0), c_mar = __shfl_sync(kFull, rc, 1);
+  const float inv_st = __shfl_sync(kFull, rc, 2);
+  const float e2 = __shfl_sync(kFull, ex, 0), e_p = __shfl_sync(kFull, ex, 2), e_q = __shfl_sync(kFull, ex, 3);
+  const float sc_d = __shfl_sync(kFull, ex, 4), sc_t = __shfl_sync(kFull, ex, 5);
+  float C = 0.f;
+  unsigned long long cfx = 0ull;
+  const float qscale = sc_d * inv_s;                            // 2^(res_m) / s
+  if (HAS_D) {
+    // H = -sum p ln p = ln2 (log2 s - t2 / s)                      (Sec. III.B(1))
+    const float l2s = log2_split(d.s);
+    const float H = kLn2 * (l2s - d.t2 * inv_s);
+    // P(1) - P(2) = (1 - e^(z(2) - m)) / sum e^(z - m)
+    const float psm = (1.0f - e2) * qscale;
+    const float c_ent = 1.0f - H * a.inv_log_v;
+    const float c_soft = psm * a.soft_norm;
+    float hi, lo;
+    dot3_exact(a.lam0, c_ent, a.lam1, c_mar, a.lam2, c_soft, hi, lo);
+    if (hi + lo >= 1.0f) { C = 1.0f; cfx = 1ull << kFixedShift; }
+    else if (hi + lo <= 0.0f) { C = 0.0f; cfx = 0ull; }
+    else {
+      C = hi;
+      const long long f = __float2ll_rn(hi * kFixedScale) + __float2ll_rn(lo * kFixedScale);
+      cfx = f < 0 ? 0ull : (unsigned long long)f;
+    }
+    if (lane == 0) {
+      if (a.H) a.H[r] = H;
+      if (a.margin) a.margin[r] = margin;
+      if (a.argmax) a.argmax[r] = d.idx;
+      if (a.conf) a.conf[r] = C;
+      // ln sum e^z = m + ln2 (log2 s - res_m)
+      if (a.lse) a.lse[r] = d.m + kLn2 * (l2s - res_m);
+    }
+  } else {
+    C = __ldg(a.conf_in + r);
+    cfx = __float2ull_rn(fminf(1.0f, fmaxf(0.0f, C)) * kFixedScale);
+  }
+  bool acc = false;
+  if (HAS_T) {
+    // Sec. III.B(c): tau_t = tau_base + gamma (1 - C_t) (tau_sign = -1: + gamma C_t)
+    const float tau = (a.tau_sign >= 0) ? fmaf(a.gamma, 1.0f - C, a.tau_base) : fmaf(a.gamma, C, a.tau_base);
+    const bool rank_ok = a.beta_rank <= 0 || t.cnt < a.beta_rank;
+    if (!SAMPLED) {
+      // gap-bounded acceptance: log P(y1) - log P(draft) = M - z_draft <= tau
+      acc = rank_ok && (t.m - c_tgt <= tau);
+      if (lane == 0 && !acc) a.out_tokens[(size_t)b * a.Ko + i] = t.idx;   // the correction, if first failure
+    } else {
+      const float p = e_p * sc_t * inv_st;                      // e^(c - M) / sum e^(z - M)
+      const float q = MODE == kModeVerify ? e_q : e_q * qscale;
+      const U4 w = philox4x32_10(U4{0u, (uint32_t)b, (uint32_t)i, iter_word(a.iteration, kPurposeAccept)},
+                                 seed_lo(a.seed), seed_hi(a.seed));
+      acc = rank_ok && (word_to_unit(w.x) * q < expf(tau) * p);
+      if (lane == 0) {
+        float MLd = MLd0, Sd = d.s;
+        if (MODE == kModeVerify) {            // q_v = 2^(z log2e - MLd) / Sd with MLd = lse log2e
+          MLd = lse_in * kLog2e;
+          Sd = exp2f(fmaf(lse_in, kLog2e, -MLd));
+        }
+        W.row_dstat[r] = make_float2(MLd, Sd);
+        W.row_tstat[r] = make_float2(MLt, t.s);
+      }
+    }
+    if (lane == 0) {
+      W.row_acc[r] = acc ? 1 : 0;
+      W.row_targmax[r] = t.idx;
+    }
+  }
+  if (lane == 0) W.row_conf[r] = cfx;
+  acc_out = acc;
+  cfx_out = cfx;
+}
+
+// ---------------------------------------------------------------------------
+// the streaming pass
+// ---------------------------------------------------------------------------
 
 // Running state of the segment a warp is reducing.
-template <typename T>
 struct SegState {
   DLane d;
   TLane t;
@@ -784,25 +835,20 @@ struct SegState {
   float zd;         // drafter logit at the drafted token (SAMPLED rule)
 };
 
-template <typename T, int MODE, bool SAMPLED>
-__device__ __forceinline__ void seg_begin(SegState<T>& ss, float c_tgt, float zd, int beta) {
-  dlane_init(ss.d);
-  tlane_init(ss.t, c_tgt, beta);
-  ss.c = c_tgt;
-  ss.zd = zd;
-}
-
-// End of a segment (row ar / storage row r / sequence b, position i, len
-// logits): warp-reduce, publish the partial, and merge the row / run the
-// sequence epilogue if this warp completes them.
-template <typename T, int MODE, bool SAMPLED>
-__device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, int b, int i, int len,
-                           const StreamSplit& sp, int w, int lane) {
-  const T* dp = (const T*)a.draft + (size_t)r * (size_t)a.V;
-  const T* tp = (MODE != kModeConf) ? (const T*)a.target + (size_t)r * (size_t)a.V : nullptr;
+// End of a segment (row ar, position r = b*K + i, len logits): warp-reduce,
+// publish the partial, and merge the row / run the sequence epilogue if this
+// warp completes them.
+template <typename T, int MODE, bool SAMPLED, bool PH2>
+__device__ void seg_finish(const StreamArgs& a, SegState& ss, int ar, int r, int b, int i, int len,
+                           const StreamSplit& sp, int w, int lane, const T* dp, const T* tp) {
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   const Workspace& W = a.ws;
+  // every lane requests the 16-byte vector in which its own maximum first
+  // appeared before the warp reductions, so the load overlaps the shuffles
+  uint4 dq = make_uint4(0, 0, 0, 0), tq = make_uint4(0, 0, 0, 0);
+  if (HAS_D && ss.d.posw > 1) dq = __ldcg(reinterpret_cast<const uint4*>(dp + ss.d.pos));
+  if (HAS_T && ss.t.posw > 1) tq = __ldcg(reinterpret_cast<const uint4*>(tp + ss.t.pos));
   DRed dr = dred_empty();
   TRed tr = tred_empty();
   if (HAS_D) {
@@ -816,15 +862,17 @@ __device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, 
     }
     float s, t2;
     d_final(d, s, t2);
-    // only lanes holding the segment maximum resolve their exact index
-    const float M = warp_max(d.m);
-    const int idx = (d.m == M && d.posw) ? first_equal<T>(dp, d.pos, d.posw, d.m, true) : kIntMax;
-    dr = reduce_d(DRed{d.m, s, t2, top2, idx});
+    const float me = d_mexp(d);
+    const float M = warp_max(me);
+    int idx = kIntMax;
+    if (me == M && d.posw) idx = d.posw > 1 ? d.pos + first_in_vec<T>(dq, me, true) : d.pos;
+    dr = reduce_d(DRed{me, s, t2, top2, idx});
   }
   if (HAS_T) {
     const TLane& t = ss.t;
     const float M = warp_max(t.M);
-    const int idx = (t.M == M && t.posw) ? first_equal<T>(tp, t.pos, t.posw, t.M, false) : kIntMax;
+    int idx = kIntMax;
+    if (t.M == M && t.posw) idx = t.posw > 1 ? t.pos + first_in_vec<T>(tq, t.M, false) : t.pos;
     tr = reduce_t(TRed{t.M, SAMPLED ? t_final(t) : 0.f, idx, t.cnt});
   }
   // lane 0 stores the partial and counts it with a release; the warp that
@@ -843,6 +891,11 @@ __device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, 
   if (old + len != a.V) return;
   // -- this warp completed row r: merge every slice's partial -----------------
   __syncwarp();
+  const int kb = k_of(a, b);
+  const bool packed = a.K <= kPackedMaxK;
+  // the drafted tokens of the window, needed if this row completes the sequence
+  int tok = -1;
+  if (HAS_T && packed && lane < kb) tok = __ldg(a.tokens + b * a.K + lane);
   const int wf = sp.first_warp(ar);
   const int wl = sp.last_warp(ar);
   DRed dm = dred_empty();
@@ -855,17 +908,35 @@ __device__ void seg_finish(const StreamArgs& a, SegState<T>& ss, int ar, int r, 
   }
   if (HAS_D) dr = reduce_d(dm);
   if (HAS_T) tr = reduce_t(tm);
-  const int kb = k_of(a, b);
-  int sold = 0;
-  if (lane == 0) {
-    W.row_done[r] = 0;
-    row_results<T, MODE, SAMPLED>(a, r, b, i, dr, tr, ss.c, ss.zd);
-    sold = atom_add_acq_rel(W.seq_done + b, 1);
-  }
-  sold = __shfl_sync(kFull, sold, 0);
-  if (sold + 1 == kb) {
-    __syncwarp();
-    seq_epilogue<MODE, SAMPLED>(a, b, kb, lane);
+  if (packed) {
+    unsigned long long word = 0ull;
+    bool acc;
+    unsigned long long cfx;
+    row_results<T, MODE, SAMPLED>(a, r, b, i, dr, tr, ss.c, ss.zd, lane, acc, cfx);
+    if (lane == 0) {
+      W.row_done[r] = 0;
+      const unsigned long long mine = 1ull | ((unsigned long long)(acc ? 1u : 0u) << (6 + i)) | (cfx << 22);
+      word = atom_add_acq_rel_u64(W.seq_word + b, mine) + mine;
+    }
+    word = __shfl_sync(kFull, word, 0);
+    if ((int)(word & 63ull) == kb) {
+      __syncwarp();
+      seq_epilogue_packed<MODE, SAMPLED, PH2>(a, b, kb, word, tok, lane);
+    }
+  } else {
+    int sold = 0;
+    bool acc;
+    unsigned long long cfx;
+    row_results<T, MODE, SAMPLED>(a, r, b, i, dr, tr, ss.c, ss.zd, lane, acc, cfx);
+    if (lane == 0) {
+      W.row_done[r] = 0;
+      sold = atom_add_acq_rel(W.seq_done + b, 1);
+    }
+    sold = __shfl_sync(kFull, sold, 0);
+    if (sold + 1 == kb) {
+      __syncwarp();
+      seq_epilogue_loads<MODE, SAMPLED, PH2>(a, b, kb, lane);
+    }
   }
 }
 
@@ -894,7 +965,7 @@ __device__ __forceinline__ void pipe_start(Pipe<T>& p, const T* dp, const T* tp,
   const int nvec = (vb - va) / VEC;
   p.nt = nvec > lane ? (nvec - lane + 31) / 32 : 0;
   p.nst = (nvec + 32 * U - 1) / (32 * U);
-  p.gd = reinterpret_cast<const uint4*>(dp + va) + lane;
+  p.gd = HAS_D ? reinterpret_cast<const uint4*>(dp + va) + lane : nullptr;
   p.gt = HAS_T ? reinterpret_cast<const uint4*>(tp + va) + lane : nullptr;
 #pragma unroll
   for (int u = 0; u < U; ++u) {
@@ -906,7 +977,7 @@ __device__ __forceinline__ void pipe_start(Pipe<T>& p, const T* dp, const T* tp,
 }
 
 template <typename T, int MODE, bool SAMPLED>
-__device__ __forceinline__ void pipe_run(Pipe<T>& p, SegState<T>& ss, int va, int beta, int lane) {
+__device__ __forceinline__ void pipe_run(Pipe<T>& p, SegState& ss, int va, int beta, int lane) {
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   constexpr int VEC = Elem<T>::kVec;
@@ -922,14 +993,34 @@ __device__ __forceinline__ void pipe_run(Pipe<T>& p, SegState<T>& ss, int va, in
       }
     }
     const int t0 = s * U;
+    // maximum phase: running maxima, top-2, rank count
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       if (t0 + u < p.nt) {
         const int v = va + (lane + 32 * (t0 + u)) * VEC;
-        if (HAS_D) d_vec(ss.d, as_vec<T>(p.d[u]), v);
-        if (HAS_T) t_vec<SAMPLED>(ss.t, as_vec<T>(p.t[u]), v, ss.c, beta);
+        if (HAS_D) d_vmax(ss.d, as_vec<T>(p.d[u]), v);
+        if (HAS_T) t_vmax(ss.t, as_vec<T>(p.t[u]), v, ss.c, beta);
       }
     }
+    // one reference check per stage, then the stage's exponentials
+    if (HAS_D) {
+      const float me = d_mexp(ss.d);
+      if (me > ss.d.ref + kRefSlack) d_reref(ss.d, me);
+    }
+    if (HAS_T && SAMPLED && ss.t.M > ss.t.ref + kRefSlack) t_reref(ss.t, ss.t.M);
+    u64 ds = 0ull, dt = 0ull, ts = 0ull;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (t0 + u < p.nt) {
+        if (HAS_D) d_vexp(ss.d, as_vec<T>(p.d[u]), ds, dt);
+        if (HAS_T && SAMPLED) t_vexp(ss.t, as_vec<T>(p.t[u]), ts);
+      }
+    }
+    if (HAS_D) {
+      kahan(ss.d.s, ss.d.cs, lo32f(ds) + hi32f(ds));
+      kahan(ss.d.t, ss.d.ct, lo32f(dt) + hi32f(dt));
+    }
+    if (HAS_T && SAMPLED) kahan(ss.t.s, ss.t.cs, lo32f(ts) + hi32f(ts));
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       if (HAS_D) p.d[u] = nd[u];
@@ -942,7 +1033,7 @@ __device__ __forceinline__ void pipe_run(Pipe<T>& p, SegState<T>& ss, int va, in
 // Order of a segment's start: its first stage of logits is requested, then
 // the logits at its drafted token (whose index was requested one segment
 // earlier), so the slice's first loads are not held up behind the token.
-template <typename T, int MODE, bool SAMPLED>
+template <typename T, int MODE, bool SAMPLED, bool PH2>
 __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_begin, int64_t e_end,
                            const StreamSplit& sp, int w, int lane) {
   constexpr bool HAS_D = MODE != kModeVerify;
@@ -950,29 +1041,31 @@ __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_beg
   const int beta = a.beta_rank > 0 ? a.beta_rank : 0;
   const void* base = HAS_D ? a.draft : a.target;
   int tok_next = 0;
-  if (HAS_T) tok_next = __ldg(a.tokens + make_seg<T>(a, s_pref, e_begin, e_end, base).r);
+  if (HAS_T) tok_next = __ldg(a.tokens + make_seg<T>(a, s_pref, e_begin, e_end, base, !HAS_D).r);
   for (int64_t e0 = e_begin; e0 < e_end;) {
-    const Seg sg = make_seg<T>(a, s_pref, e0, e_end, base);
+    const Seg sg = make_seg<T>(a, s_pref, e0, e_end, base, !HAS_D);
     const int len = sg.v1 - sg.v0;
     e0 += len;
-    const size_t rowoff = (size_t)sg.r * (size_t)a.V;
-    const T* dp = (const T*)a.draft + rowoff;
-    const T* tp = HAS_T ? (const T*)a.target + rowoff : nullptr;
+    const T* dp = (const T*)a.draft + (size_t)sg.r * (size_t)a.V;
+    const T* tp = HAS_T ? (const T*)a.target + ((size_t)sg.b * a.Kt + sg.i) * (size_t)a.V : nullptr;
     Pipe<T> pp;
     pipe_start<T, MODE>(pp, dp, tp, sg.va, sg.vb, lane);
     float c = 0.f, zd = 0.f;
     if (HAS_T) {
       int tok = tok_next;
-      if (e0 < e_end) tok_next = __ldg(a.tokens + make_seg<T>(a, s_pref, e0, e_end, base).r);
-      if (tok < 0 || tok >= a.V) {
+      if (e0 < e_end) tok_next = __ldg(a.tokens + make_seg<T>(a, s_pref, e0, e_end, base, !HAS_D).r);
+      if (tok < 0 || tok >= a.V) {       // out-of-range draft: clamped, reported
         if (lane == 0) atomicOr(a.ws.err, 1u);
         tok = 0;
       }
       c = Elem<T>::load(tp + tok);
       if (SAMPLED) zd = Elem<T>::load(dp + tok);
     }
-    SegState<T> ss;
-    seg_begin<T, MODE, SAMPLED>(ss, c, zd, beta);
+    SegState ss;
+    dlane_init(ss.d);
+    tlane_init(ss.t, c, beta);
+    ss.c = c;
+    ss.zd = zd;
     if (lane < sg.va - sg.v0) {
       const int v = sg.v0 + lane;
       if (HAS_D) d_scalar(ss.d, Elem<T>::load(dp + v), v);
@@ -984,25 +1077,405 @@ __device__ void walk_slice(const StreamArgs& a, const int* s_pref, int64_t e_beg
       if (HAS_D) d_scalar(ss.d, Elem<T>::load(dp + v), v);
       if (HAS_T) t_scalar<SAMPLED>(ss.t, Elem<T>::load(tp + v), v, ss.c, beta);
     }
-    seg_finish<T, MODE, SAMPLED>(a, ss, sg.ar, sg.r, sg.b, sg.i, len, sp, w, lane);
+    seg_finish<T, MODE, SAMPLED, PH2>(a, ss, sg.ar, sg.r, sg.b, sg.i, len, sp, w, lane, dp, tp);
   }
 }
 
-template <typename T, int MODE, bool SAMPLED>
-__global__ void __launch_bounds__(kStreamThreads, CMSD_MIN_BLOCKS) stream_kernel(const StreamArgs a) {
+// ---------------------------------------------------------------------------
+// second pass: the residual draw and the bonus token (resample kernel)
+// ---------------------------------------------------------------------------
+//
+// The residual draw at a rejected position is a two-level exponential race
+// over r_v = max(0, p_v - q_v).  Level 1 races the groups of kGroup
+// consecutive entries on their masses R_g = sum of r_v (key E_g / R_g,
+// E_g = -log(1-U_g)); level 2 races the entries of the winning group (key
+// E_v / r_v).  The group wins with probability R_g / R and the entry within
+// it with r_v / R_g, so the token has the law r_v / R of the normalised
+// residual.  The bonus token under the sampled rule is the same race with
+// r = p; under the PAPER rule it is the verifier row's argmax.
+//
+// Work is split over warps in units of (queued row, group); a warp walks its
+// groups one shared-memory stage at a time (all of a stage's loads in flight
+// together, cp.async), GPI groups per iteration, LPG lanes per group with one
+// 16-byte vector each.  A group is raced (logarithm and division) only when
+// its uniform passes a bound against the warp's best key so far.  Each warp's
+// best (key, group) goes to a partial slot with its level-2 winner; the warp
+// that completes a row merges the partials.
+
+// r = max(0, p - q), p = e^(zt - Mt) / St, q = e^(zd - Md) / Sd, with every
+// operation rounded on its own (p - q formed as p + (-q)), so that the packed
+// form below gives the same bits per entry.
+struct RowStat {
+  float MLt, invSt;    // verifier: max*log2e, 1 / sum
+  float MLd, ninvSd;   // drafter: max*log2e, -1 / sum (0: no drafter term)
+};
+
+__device__ __forceinline__ float resid(float zt, float zd, const RowStat& s) {
+  const float p = __fmul_rn(ex2(__fmaf_rn(zt, kLog2e, -s.MLt)), s.invSt);
+  const float qn = __fmul_rn(ex2(__fmaf_rn(zd, kLog2e, -s.MLd)), s.ninvSd);
+  return fmaxf(__fadd_rn(p, qn), 0.f);
+}
+
+__device__ __forceinline__ float expo(uint32_t word) { return -log1pf(-word_to_unit(word)); }
+
+// resid() of two entries at once (packed f32x2), accumulated into acc.
+__device__ __forceinline__ void resid2(u64& acc, u64 zt, u64 zd, const RowStat& s) {
+  const u64 p = mul2(ex2_2(fma2(zt, dup2(kLog2e), dup2(-s.MLt))), dup2(s.invSt));
+  const u64 qn = mul2(ex2_2(fma2(zd, dup2(kLog2e), dup2(-s.MLd))), dup2(s.ninvSd));
+  const u64 r = add2(p, qn);
+  acc = add2(acc, pack2(fmaxf(lo32f(r), 0.f), fmaxf(hi32f(r), 0.f)));
+}
+
+// Sum of r over the entries of one 16-byte vector pair.
+template <typename T>
+__device__ __forceinline__ float resid_vec(uint4 qt, uint4 qd, const RowStat& s) {
+  u64 acc = 0ull;
+  if (sizeof(T) == 2) {
+    resid2(acc, bf2_to_f2(qt.x), bf2_to_f2(qd.x), s);
+    resid2(acc, bf2_to_f2(qt.y), bf2_to_f2(qd.y), s);
+    resid2(acc, bf2_to_f2(qt.z), bf2_to_f2(qd.z), s);
+    resid2(acc, bf2_to_f2(qt.w), bf2_to_f2(qd.w), s);
+  } else {
+    resid2(acc, pack2(__uint_as_float(qt.x), __uint_as_float(qt.y)),
+           pack2(__uint_as_float(qd.x), __uint_as_float(qd.y)), s);
+    resid2(acc, pack2(__uint_as_float(qt.z), __uint_as_float(qt.w)),
+           pack2(__uint_as_float(qd.z), __uint_as_float(qd.w)), s);
+  }
+  return lo32f(acc) + hi32f(acc);
+}
+
+// 16 bytes of logits at entry v of one row: one vector load when the vector is
+// aligned and inside the row, else element loads with entries past the row
+// end read as -inf (p = q = 0, so r = 0).
+template <typename T>
+__device__ __forceinline__ uint4 load_logits(const T* p, int v, int V, bool vec_ok) {
+  constexpr int VEC = Elem<T>::kVec;
+  if (vec_ok && v + VEC <= V) return __ldcg(reinterpret_cast<const uint4*>(p + v));
+  uint32_t w[4];
+  if (sizeof(T) == 2) {
+    const unsigned short* q = reinterpret_cast<const unsigned short*>(p);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint32_t lo = (v + 2 * k < V) ? (uint32_t)__ldg(q + v + 2 * k) : 0xFF80u;
+      const uint32_t hi = (v + 2 * k + 1 < V) ? (uint32_t)__ldg(q + v + 2 * k + 1) : 0xFF80u;
+      w[k] = lo | (hi << 16);
+    }
+  } else {
+    const uint32_t* q = reinterpret_cast<const uint32_t*>(p);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) w[k] = (v + k < V) ? __ldg(q + v + k) : 0xFF800000u;
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+template <typename T>
+__device__ __forceinline__ uint4 neg_inf_vec() {
+  return sizeof(T) == 2 ? make_uint4(kNegInf2, kNegInf2, kNegInf2, kNegInf2)
+                        : make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
+}
+
+// Level 2 on group gm, whose logits sit in lanes own .. own+LPG-1 (vector
+// `sub` of the group in lane own+sub): every lane takes one entry, gathers its
+// logit pair by shuffles and races E_v / r_v.  Returns the warp's least key
+// (lowest entry on ties) as the entry index, or -1 if no entry has r_v > 0.
+template <typename T>
+__device__ __forceinline__ int race_group_entries(uint4 qt, uint4 qd, int gm, int own, int lane,
+                                                  const RowStat& st, uint32_t b, uint32_t n,
+                                                  uint32_t cw, uint32_t k0, uint32_t k1) {
+  constexpr int VEC = Elem<T>::kVec;
+  const int src = own + lane / VEC;
+  const int k = lane % VEC;
+  const uint32_t t0 = __shfl_sync(kFull, qt.x, src), t1 = __shfl_sync(kFull, qt.y, src);
+  const uint32_t t2 = __shfl_sync(kFull, qt.z, src), t3 = __shfl_sync(kFull, qt.w, src);
+  const uint32_t d0 = __shfl_sync(kFull, qd.x, src), d1 = __shfl_sync(kFull, qd.y, src);
+  const uint32_t d2 = __shfl_sync(kFull, qd.z, src), d3 = __shfl_sync(kFull, qd.w, src);
+  const float zt = logit_at<T>(make_uint4(t0, t1, t2, t3), k);
+  const float zd = logit_at<T>(make_uint4(d0, d1, d2, d3), k);
+  const int v = gm * kGroup + lane;
+  const float rv = resid(zt, zd, st);
+  const U4 wd = philox4x32_10(U4{(uint32_t)v >> 2, b, n, cw}, k0, k1);
+  const uint32_t sel = (uint32_t)v & 3u;
+  const uint32_t word = sel == 0 ? wd.x : sel == 1 ? wd.y : sel == 2 ? wd.z : wd.w;
+  const float key = rv > 0.f ? expo(word) / rv : pos_inf();
+  const float km = warp_min(key);
+  const int vm = warp_min_i(key == km ? v : kIntMax);
+  return km != pos_inf() ? vm : -1;
+}
+
+#ifndef CMSD_RES_MIN_BLOCKS
+#define CMSD_RES_MIN_BLOCKS 3
+#endif
+constexpr int kGroupBatch = 128;       // group uniforms one warp draws at once (4 per lane)
+constexpr int kResMinGroups = 48;      // fewest groups per warp
+constexpr int kResStageBytes = 8192;   // shared-memory stage per warp (both tensors)
+constexpr float kRaceFilter = 0.99999f;  // 1 - 1e-5
+constexpr size_t kResSmemBytes = (size_t)kResWarps * kResStageBytes;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+// The groups [gc, ge) of one row (target, and drafter when `two`) into this
+// warp's stage: the vectors wholly inside the row go by cp.async, all in
+// flight together; returns how many (the rest is read element by element).
+template <typename T>
+__device__ __forceinline__ int stage_groups(const T* tp, const T* dp, bool two, int gc, int ge, int V, bool vec_ok,
+                                            uint32_t st_t, uint32_t st_d, int lane) {
+  constexpr int VEC = Elem<T>::kVec;
+  constexpr int LPG = kGroup / VEC;
+  const int v_base = gc * kGroup;
+  const int nfull = vec_ok ? min((ge - gc) * LPG, (V - v_base) / VEC) : 0;
+  for (int j = lane; j < nfull; j += 32) {
+    cp_async16(st_t + 16u * (uint32_t)j, tp + v_base + j * VEC);
+    if (two) cp_async16(st_d + 16u * (uint32_t)j, dp + v_base + j * VEC);
+  }
+  cp_async_commit();
+  cp_async_wait_all();
+  __syncwarp();
+  return nfull;
+}
+
+// Vector `sub` of group g (staged chunk starting at group gc), or -inf
+// padding past the row end.
+template <typename T>
+__device__ __forceinline__ uint4 staged_vec(const unsigned char* stage, const T* row, int g, int gc, int ge, int sub,
+                                            int nfull, int V) {
+  constexpr int VEC = Elem<T>::kVec;
+  constexpr int LPG = kGroup / VEC;
+  if (g >= ge) return neg_inf_vec<T>();
+  const int j = (g - gc) * LPG + sub;
+  if (j < nfull) return *reinterpret_cast<const uint4*>(stage + 16 * j);
+  return load_logits<T>(row, g * kGroup + sub * VEC, V, false);
+}
+
+template <typename T, bool SAMPLED>
+__global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_kernel(const StreamArgs a) {
+  constexpr int VEC = Elem<T>::kVec;
+  constexpr int LPG = kGroup / VEC;    // lanes per group
+  constexpr int GPI = 32 / LPG;        // groups per warp iteration
+  constexpr int CG = kResStageBytes / (2 * kGroup * (int)sizeof(T));   // groups per stage
+  extern __shared__ __align__(16) unsigned char res_smem[];
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const unsigned char* stage = res_smem + warp * kResStageBytes;
+  const uint32_t st_t = smem_u32(stage), st_d = st_t + kResStageBytes / 2;
+  // everything below reads what the streaming kernel wrote: wait until that
+  // grid has completed and its memory is visible
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const Workspace& W = a.ws;
+  int R = __ldcg(W.rec_count);
+  R = R < 0 ? 0 : (R > a.B ? a.B : R);
+  const int ng = (a.V + kGroup - 1) / kGroup;
+  const int64_t NU = (int64_t)R * ng;
+  if (NU > 0) {
+    int64_t want = NU / kResMinGroups;
+    const int Weff = (int)(want < 1 ? 1 : (want > a.nwarps ? a.nwarps : want));
+    const int w = blockIdx.x * kResWarps + warp;
+    if (w < Weff) {
+      const EvenSplit sp(NU, Weff);
+      int64_t u0 = sp.start(w);
+      const int64_t u1 = sp.start(w + 1);
+      const uint32_t k0 = seed_lo(a.seed), k1 = seed_hi(a.seed);
+      const uint32_t cw_grp = iter_word(a.iteration, kPurposeGroup);
+      const uint32_t cw_ent = iter_word(a.iteration, kPurposeResidual);
+      const int sub = lane % LPG;
+      while (u0 < u1) {
+        const int rr = (int)div_nn(u0, ng);
+        const int g0 = (int)(u0 - (int64_t)rr * ng);
+        const int cnt = (int)min((int64_t)(ng - g0), u1 - u0);
+        const int g1 = g0 + cnt;
+        const int4 rec = __ldcg(W.rec + rr);
+        const int b = rec.x, pos = rec.y, kind = rec.z;
+        const int r = b * a.K + pos;                                   // position (stats)
+        const T* tp = (const T*)a.target + ((size_t)b * a.Kt + pos) * (size_t)a.V;
+        const bool resid_kind = SAMPLED && kind == kSeqResidual;
+        const T* dp = resid_kind ? (const T*)a.draft + (size_t)r * (size_t)a.V : tp;
+        const bool vec_ok = ((((uintptr_t)tp) | ((uintptr_t)dp)) & 15) == 0;
+        float2 ts = make_float2(0.f, 1.f), ds = make_float2(0.f, 1.f);
+        if (resid_kind) {
+          ts = __ldcg(W.row_tstat + r);
+          ds = __ldcg(W.row_dstat + r);
+        }
+        UnitResult res;
+        res.key = pos_inf();
+        res.ref = 0.f;
+        res.grp = kIntMax;
+        res.tok = -1;
+        if (!SAMPLED) {
+          // PAPER rule, bonus row: the warp's largest logit (lowest index); key = -max
+          float best = -pos_inf();
+          int bi = kIntMax;
+          for (int gc = g0; gc < g1; gc += CG) {
+            const int ge = min(g1, gc + CG);
+            const int nfull = stage_groups<T>(tp, dp, false, gc, ge, a.V, vec_ok, st_t, st_d, lane);
+            for (int gi = gc; gi < ge; gi += GPI) {
+              const int g = gi + lane / LPG;
+              const uint4 qt = staged_vec<T>(stage, tp, g, gc, ge, sub, nfull, a.V);
+              const int v = g * kGroup + sub * VEC;
+#pragma unroll
+              for (int k = 0; k < VEC; ++k) {
+                const float z = logit_at<T>(qt, k);
+                if (z > best) { best = z; bi = v + k; }
+              }
+            }
+            __syncwarp();
+          }
+          const float mx = warp_max(best);
+          const int im = warp_min_i(best == mx ? bi : kIntMax);
+          if (mx != -pos_inf()) {
+            res.key = -mx;
+            res.grp = im;
+            res.tok = im;
+          }
+        } else {
+          RowStat st{0.f, 1.0f, 0.f, 0.f};   // the residual's is formed once the first stage is in
+          if (!resid_kind) {
+            // bonus race over p: terms relative to the warp's largest logit (a first pass)
+            float mx = -pos_inf();
+            for (int v = g0 * kGroup + lane * VEC; v < g1 * kGroup && v < a.V; v += 32 * VEC) {
+              const uint4 q = load_logits<T>(tp, v, a.V, vec_ok);
+#pragma unroll
+              for (int k = 0; k < VEC; ++k) mx = fmaxf(mx, logit_at<T>(q, k));
+            }
+            mx = warp_max(mx);
+            res.ref = mx == -pos_inf() ? 0.f : mlog2e(mx);
+            st = RowStat{res.ref, 1.0f, 0.f, 0.f};
+          }
+          float best = pos_inf();              // this lane set's least key
+          float thr = pos_inf();               // the warp's least key so far (filter bound)
+          int bestg = kIntMax;
+          uint4 bqt = neg_inf_vec<T>(), bqd = make_uint4(0, 0, 0, 0);
+          int gb = -kGroupBatch;               // first group of the drawn batch
+          U4 gw = U4{0u, 0u, 0u, 0u};
+          for (int gc = g0; gc < g1; gc += CG) {
+            const int ge = min(g1, gc + CG);
+            const int nfull = stage_groups<T>(tp, dp, resid_kind, gc, ge, a.V, vec_ok, st_t, st_d, lane);
+            if (resid_kind && gc == g0) st = RowStat{ts.x, 1.0f / ts.y, ds.x, -1.0f / ds.y};
+            for (int gi = gc; gi < ge; gi += GPI) {
+              const int g = gi + lane / LPG;
+              const uint4 qt = staged_vec<T>(stage, tp, g, gc, ge, sub, nfull, a.V);
+              const uint4 qd = resid_kind ? staged_vec<T>(stage + kResStageBytes / 2, dp, g, gc, ge, sub, nfull, a.V)
+                                          : make_uint4(0, 0, 0, 0);
+              if (gi + GPI > gb + kGroupBatch) {   // warp-uniform: draw the next 128 group uniforms
+                gb = gi & ~3;
+                gw = philox4x32_10(U4{(uint32_t)(gb >> 2) + (uint32_t)lane, (uint32_t)b, (uint32_t)pos, cw_grp},
+                                   k0, k1);
+              }
+              float acc = resid_vec<T>(qt, qd, st);
+#pragma unroll
+              for (int o = 1; o < LPG; o <<= 1) acc += __shfl_xor_sync(kFull, acc, o);
+              const int off = min(g - gb, kGroupBatch - 1);
+              const int src = off >> 2, sel = off & 3;
+              const uint32_t x0 = __shfl_sync(kFull, gw.x, src), x1 = __shfl_sync(kFull, gw.y, src);
+              const uint32_t x2 = __shfl_sync(kFull, gw.z, src), x3 = __shfl_sync(kFull, gw.w, src);
+              const uint32_t word = sel == 0 ? x0 : sel == 1 ? x1 : sel == 2 ? x2 : x3;
+              // E_g >= U_g, so a group with U_g >= thr R_g has a key above the
+              // warp's best so far and cannot win (the factor covers the
+              // rounding of E and of the product)
+              bool improved = false;
+              if (g < ge && acc > 0.f && word_to_unit(word) * kRaceFilter < thr * acc) {
+                const float key = expo(word) / acc;
+                if (key < best) {          // groups are visited in increasing order
+                  best = key;
+                  bestg = g;
+                  bqt = qt;
+                  bqd = qd;
+                  improved = true;
+                }
+              }
+              if (__any_sync(kFull, improved)) thr = warp_min(best);
+            }
+            __syncwarp();                  // the stage is rewritten by the next chunk
+          }
+          const float kmin = warp_min(best);
+          const int gmin = warp_min_i(best == kmin ? bestg : kIntMax);
+          if (kmin != pos_inf()) {
+            // level 2 on this warp's winning group (its lanes hold it as their best)
+            const int own = ((gmin - g0) % GPI) * LPG;
+            res.tok = race_group_entries<T>(bqt, bqd, gmin, own, lane, st, (uint32_t)b, (uint32_t)pos, cw_ent,
+                                            k0, k1);
+            res.key = kmin;
+            res.grp = gmin;
+          }
+        }
+        int old = 0;
+        if (lane == 0) {
+          W.rpart[rr + w] = res;
+          old = atom_add_acq_rel(W.res_done + rr, cnt);
+        }
+        old = __shfl_sync(kFull, old, 0);
+        if (old + cnt == ng) {
+          // this warp completed row rr: merge the partials of the warps that covered it
+          __syncwarp();
+          const int wf = sp.owner((int64_t)rr * ng);
+          const int wl = sp.owner((int64_t)rr * ng + ng - 1);
+          const bool bonus_race = SAMPLED && kind == kSeqBonus;
+          float rmax = -pos_inf();
+          if (bonus_race) {
+            for (int k = wf + lane; k <= wl; k += 32) rmax = fmaxf(rmax, __ldcg(&W.rpart[rr + k].ref));
+            rmax = warp_max(rmax);
+          }
+          float key = pos_inf();
+          int gw_ = kIntMax, tw = -1;
+          for (int k = wf + lane; k <= wl; k += 32) {
+            const int4 x = __ldcg(reinterpret_cast<const int4*>(W.rpart + rr + k));
+            float xk = __int_as_float(x.x);
+            // bonus race: a warp's key is relative to its own reference: key * 2^(rmax - ref)
+            if (bonus_race && xk != pos_inf()) xk *= exp2_diff(rmax, __int_as_float(x.y));
+            if (xk < key || (xk == key && x.z < gw_)) {
+              key = xk;
+              gw_ = x.z;
+              tw = x.w;
+            }
+          }
+          const float km = warp_min(key);
+          const int gm = warp_min_i(key == km ? gw_ : kIntMax);
+          const int tm = warp_min_i((key == km && gw_ == gm && tw >= 0) ? tw : kIntMax);
+          if (lane == 0) {
+            W.res_done[rr] = 0;
+            int out = tm;
+            if (gm == kIntMax || tm == kIntMax) out = __ldcg(W.row_targmax + r);   // empty residual: argmax
+            a.out_tokens[(size_t)b * a.Ko + pos] = out;
+          }
+        }
+        u0 += cnt;
+      }
+    }
+  }
+  // the last CTA to finish clears the queue for the next call
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int done = atom_add_acq_rel(W.res_cta_done, 1);
+    if (done == (int)gridDim.x - 1) {
+      *W.rec_count = 0;
+      *W.res_cta_done = 0;
+      __threadfence();
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// the kernel
+// ---------------------------------------------------------------------------
+
+template <typename T, int MODE, bool SAMPLED, bool PH2>
+__global__ void __launch_bounds__(kStreamThreads, 1) stream_kernel(const StreamArgs a) {
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   constexpr int VEC = Elem<T>::kVec;
   extern __shared__ __align__(128) unsigned char smem[];
-  // the resample kernel (launched as a programmatic dependent) may be
-  // scheduled now; it waits for this grid's completion before reading anything
-  if (SAMPLED) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
+  const int w = blockIdx.x * kStreamWarps + warp;
   const Workspace& W = a.ws;
   const bool ragged = a.k_row != nullptr;
   int* s_pref = reinterpret_cast<int*>(smem);
+  // the resample kernel (launched as a programmatic dependent) may be
+  // scheduled now; it waits for this grid's completion before reading anything
+  if (PH2) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   // -- present rows: exclusive prefix of k_row (ragged windows) -------------
   int nrows;
@@ -1042,331 +1515,85 @@ __global__ void __launch_bounds__(kStreamThreads, CMSD_MIN_BLOCKS) stream_kernel
       const int raw = __ldg(a.k_row + b);
       if (raw < 0 || raw > a.K) atomicOr(W.err, 2u);
       if (k_of(a, b) == 0) {
-        if (HAS_D && a.k_next) a.k_next[b] = a.k_min;
+        if (HAS_D && a.k_next) a.k_next[b] = a.k_fixed > 0 ? a.k_fixed : a.k_min;
         if (HAS_T) {
           a.n_accept[b] = 0;
-          for (int i = 0; i < a.K; ++i) {
-            a.out_tokens[b * a.K + i] = -1;
-            if (a.accept) a.accept[b * a.K + i] = 0;
-          }
+          for (int i = 0; i < a.Ko; ++i) a.out_tokens[(size_t)b * a.Ko + i] = -1;
+          if (a.accept)
+            for (int i = 0; i < a.K; ++i) a.accept[(size_t)b * a.K + i] = 0;
+          if (PH2) publish(a, b, a.bonus ? kSeqBonus : kSeqNone, 0);
         }
       }
     }
   }
 
-  if (nrows == 0) return;
-  const StreamSplit sp(nrows, a.V, VEC, a.nwarps, stream_min_len(a.V));
-  const int w = blockIdx.x * kStreamWarps + warp;
-  if (w >= sp.W) return;
-  const int64_t e_begin = sp.start(w);
-  const int64_t e_end = sp.start(w + 1);
-  if (e_begin >= e_end) return;
-  walk_slice<T, MODE, SAMPLED>(a, s_pref, e_begin, e_end, sp, w, lane);
-}
-
-// ---------------------------------------------------------------------------
-// residual draw at each rejected position: two-level exponential race over
-// r_v = max(0, p_v - q_v).  Level 1 races the groups of kGroup consecutive
-// entries on their masses R_g = sum of r_v (key E_g / R_g, E_g = -log(1-U_g));
-// level 2 races the entries of the winning group (key E_v / r_v).  The group
-// wins with probability R_g / R and the entry within it with r_v / R_g, so the
-// token has the law r_v / R of the normalised residual.
-//
-// Work is split over warps in units of (rejected row, group); a warp walks its
-// groups GPI at a time, LPG lanes per group with one 16-byte vector each.
-// Its best (key, group) goes to a partial slot; the warp that completes a row
-// merges the partials and runs level 2 on the winning group (one lane per
-// entry).
-// ---------------------------------------------------------------------------
-
-#ifndef CMSD_RES_MIN_BLOCKS
-#define CMSD_RES_MIN_BLOCKS 3
-#endif
-constexpr int kGroup = 32;
-constexpr int kGroupBatch = 128;       // groups whose E_g one warp draws at once (4 per lane)
-constexpr int kResMinGroups = 48;      // fewest groups per warp
-constexpr int kResStageBytes = 8192;   // shared-memory stage per warp (both tensors)
-constexpr float kRaceFilter = 0.99999f;  // 1 - 1e-5
-
-struct RowStat {
-  float MLt, invSt;    // verifier: max*log2e, 1 / sum
-  float MLd, ninvSd;   // drafter: max*log2e, -1 / sum
-};
-
-// r = max(0, p - q), p = e^(zt - Mt) / St, q = e^(zd - Md) / Sd, with every
-// operation rounded on its own (p - q formed as p + (-q), which is the same
-// rounding), so that the packed form below gives the same bits per entry.
-__device__ __forceinline__ float resid(float zt, float zd, const RowStat& s) {
-  const float p = __fmul_rn(ex2(__fmaf_rn(zt, kLog2e, -s.MLt)), s.invSt);
-  const float qn = __fmul_rn(ex2(__fmaf_rn(zd, kLog2e, -s.MLd)), s.ninvSd);
-  return fmaxf(__fadd_rn(p, qn), 0.f);
-}
-
-__device__ __forceinline__ float expo(uint32_t word) { return -log1pf(-word_to_unit(word)); }
-
-// resid() of two entries at once (packed f32x2), accumulated into acc.
-__device__ __forceinline__ void resid2(u64& acc, u64 zt, u64 zd, const RowStat& s) {
-  const u64 p = mul2(ex2_2(fma2(zt, dup2(kLog2e), dup2(-s.MLt))), dup2(s.invSt));
-  const u64 qn = mul2(ex2_2(fma2(zd, dup2(kLog2e), dup2(-s.MLd))), dup2(s.ninvSd));
-  const u64 r = add2(p, qn);
-  acc = add2(acc, pack2(fmaxf(lo32f(r), 0.f), fmaxf(hi32f(r), 0.f)));
-}
-
-// Sum of r over the entries of one 16-byte vector pair.
-template <typename T>
-__device__ __forceinline__ float resid_vec(uint4 qt, uint4 qd, const RowStat& s) {
-  u64 acc = 0ull;
-  if (sizeof(T) == 2) {
-    resid2(acc, bf2_to_f2(qt.x), bf2_to_f2(qd.x), s);
-    resid2(acc, bf2_to_f2(qt.y), bf2_to_f2(qd.y), s);
-    resid2(acc, bf2_to_f2(qt.z), bf2_to_f2(qd.z), s);
-    resid2(acc, bf2_to_f2(qt.w), bf2_to_f2(qd.w), s);
-  } else {
-    resid2(acc, pack2(__uint_as_float(qt.x), __uint_as_float(qt.y)),
-           pack2(__uint_as_float(qd.x), __uint_as_float(qd.y)), s);
-    resid2(acc, pack2(__uint_as_float(qt.z), __uint_as_float(qt.w)),
-           pack2(__uint_as_float(qd.z), __uint_as_float(qd.w)), s);
-  }
-  return lo32f(acc) + hi32f(acc);
-}
-
-
-// 16 bytes of logits at entry v of one row: one vector load when the vector is
-// aligned and inside the row, else element loads with entries past the row
-// end read as -inf (p = q = 0, so r = 0).
-template <typename T>
-__device__ __forceinline__ uint4 load_logits(const T* p, int v, int V, bool vec_ok) {
-  constexpr int VEC = Elem<T>::kVec;
-  if (vec_ok && v + VEC <= V) return ld_stream(p + v);
-  uint32_t w[4];
-  if (sizeof(T) == 2) {
-    const unsigned short* q = reinterpret_cast<const unsigned short*>(p);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const uint32_t lo = (v + 2 * k < V) ? (uint32_t)__ldg(q + v + 2 * k) : 0xFF80u;
-      const uint32_t hi = (v + 2 * k + 1 < V) ? (uint32_t)__ldg(q + v + 2 * k + 1) : 0xFF80u;
-      w[k] = lo | (hi << 16);
-    }
-  } else {
-    const uint32_t* q = reinterpret_cast<const uint32_t*>(p);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) w[k] = (v + k < V) ? __ldg(q + v + k) : 0xFF800000u;
-  }
-  return make_uint4(w[0], w[1], w[2], w[3]);
-}
-
-template <typename T>
-__device__ __forceinline__ uint4 neg_inf_vec() {
-  return sizeof(T) == 2 ? make_uint4(kNegInf2, kNegInf2, kNegInf2, kNegInf2)
-                        : make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
-}
-
-
-
-// Level 2 on group gm, whose logits sit in lanes own .. own+LPG-1 (vector
-// `sub` of the group in lane own+sub): every lane takes one entry, gathers its
-// logit pair by shuffles and races E_v / r_v.  Returns the warp's least key
-// (lowest entry on ties) as the entry index, or -1 if no entry has r_v > 0.
-template <typename T>
-__device__ __forceinline__ int race_group_entries(uint4 qt, uint4 qd, int gm, int own, int lane,
-                                                  const RowStat& st, uint32_t b, uint32_t n,
-                                                  uint32_t cw, uint32_t k0, uint32_t k1) {
-  constexpr int VEC = Elem<T>::kVec;
-  const int src = own + lane / VEC;
-  const int k = lane % VEC;
-  const uint32_t t0 = __shfl_sync(kFull, qt.x, src), t1 = __shfl_sync(kFull, qt.y, src);
-  const uint32_t t2 = __shfl_sync(kFull, qt.z, src), t3 = __shfl_sync(kFull, qt.w, src);
-  const uint32_t d0 = __shfl_sync(kFull, qd.x, src), d1 = __shfl_sync(kFull, qd.y, src);
-  const uint32_t d2 = __shfl_sync(kFull, qd.z, src), d3 = __shfl_sync(kFull, qd.w, src);
-  const float zt = logit_at<T>(make_uint4(t0, t1, t2, t3), k);
-  const float zd = logit_at<T>(make_uint4(d0, d1, d2, d3), k);
-  const int v = gm * kGroup + lane;
-  const float rv = resid(zt, zd, st);
-  const U4 wd = philox4x32_10(U4{(uint32_t)v >> 2, b, n, cw}, k0, k1);
-  const uint32_t sel = (uint32_t)v & 3u;
-  const uint32_t word = sel == 0 ? wd.x : sel == 1 ? wd.y : sel == 2 ? wd.z : wd.w;
-  const float key = rv > 0.f ? expo(word) / rv : pos_inf();
-  const float km = warp_min(key);
-  const int vm = warp_min_i(key == km ? v : kIntMax);
-  return km != pos_inf() ? vm : -1;
-}
-
-template <typename T>
-__global__ void __launch_bounds__(kThreads, CMSD_RES_MIN_BLOCKS) resample_kernel(const StreamArgs a) {
-  constexpr int VEC = Elem<T>::kVec;
-  constexpr int LPG = kGroup / VEC;    // lanes per group
-  constexpr int GPI = 32 / LPG;        // groups per warp iteration
-  constexpr int CG = kResStageBytes / (2 * kGroup * (int)sizeof(T));   // groups per chunk
-  extern __shared__ __align__(16) unsigned char res_smem[];
-  const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
-  const unsigned char* stage = res_smem + warp * kResStageBytes;
-  const uint32_t st_t = smem_u32(stage), st_d = st_t + kResStageBytes / 2;
-  // everything below reads what the streaming kernel wrote: wait until that
-  // grid has completed and its memory is visible
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  const Workspace& W = a.ws;
-  int R = __ldcg(W.rej_count);
-  R = R < 0 ? 0 : (R > a.B ? a.B : R);
-  const int ng = (a.V + kGroup - 1) / kGroup;
-  const int64_t NU = (int64_t)R * ng;
-  if (NU > 0) {
-    const int Weff = eff_warps(NU, kResMinGroups, a.nwarps);
-    const int w = blockIdx.x * kWarpsPerBlock + warp;
-    if (w < Weff) {
-      const EvenSplit sp(NU, Weff);
-      int64_t u0 = sp.start(w);
-      const int64_t u1 = sp.start(w + 1);
-      const uint32_t k0 = seed_lo(a.seed), k1 = seed_hi(a.seed);
-      const uint32_t cw_grp = iter_word(a.iteration, kPurposeGroup);
-      const uint32_t cw_ent = iter_word(a.iteration, kPurposeResidual);
-      const int sub = lane % LPG;
-      while (u0 < u1) {
-        const int rr_ = (int)div_nn(u0, ng);
-        const int g0 = (int)(u0 - (int64_t)rr_ * ng);
-        const int cnt = (int)min((int64_t)(ng - g0), u1 - u0);
-        const int g1 = g0 + cnt;
-        const int4 rq0 = __ldcg(reinterpret_cast<const int4*>(W.rej + rr_));
-        const float4 rq1 = __ldcg(reinterpret_cast<const float4*>(W.rej + rr_) + 1);
-        const int r = rq0.x, b = rq0.y, n = rq0.z;
-        const RowStat st{rq1.x, rq1.y, rq1.z, -rq1.w};
-        const size_t rowoff = (size_t)r * (size_t)a.V;
-        const T* dp = (const T*)a.draft + rowoff;
-        const T* tp = (const T*)a.target + rowoff;
-        const bool vec_ok = ((((uintptr_t)tp) | ((uintptr_t)dp)) & 15) == 0;
-
-        // level 1, one chunk of CG groups at a time: the chunk's logits are
-        // copied to this warp's shared-memory stage in one batch of cp.async
-        // (all in flight together), then raced GPI groups per iteration
-        float best = pos_inf();              // this lane set's least key
-        float thr = pos_inf();               // the warp's least key so far (filter bound)
-        int bestg = kIntMax;
-        uint4 bqt = neg_inf_vec<T>(), bqd = neg_inf_vec<T>();
-        int gb = -kGroupBatch;               // first group of the drawn batch
-        uint32_t U0 = 0, U1 = 0, U2 = 0, U3 = 0;
-        for (int gc = g0; gc < g1; gc += CG) {
-          const int ge = min(g1, gc + CG);
-          const int v_base = gc * kGroup;
-          // vectors of the chunk lying wholly inside the row (aligned rows only)
-          const int nfull = vec_ok ? min((ge - gc) * LPG, (a.V - v_base) / VEC) : 0;
-          for (int j = lane; j < nfull; j += 32) {
-            cp_async16(st_t + 16u * (uint32_t)j, tp + v_base + j * VEC);
-            cp_async16(st_d + 16u * (uint32_t)j, dp + v_base + j * VEC);
-          }
-          cp_async_commit();
-          cp_async_wait<0>();
-          __syncwarp();
-          for (int gi = gc; gi < ge; gi += GPI) {
-            const int g = gi + lane / LPG;
-            const int j = (g - gc) * LPG + sub;
-            uint4 qt = neg_inf_vec<T>(), qd = neg_inf_vec<T>();
-            if (g < ge) {
-              if (j < nfull) {
-                qt = *reinterpret_cast<const uint4*>(stage + 16 * j);
-                qd = *reinterpret_cast<const uint4*>(stage + kResStageBytes / 2 + 16 * j);
-              } else {   // ragged row end or unaligned row: element loads, -inf past the end
-                qt = load_logits<T>(tp, g * kGroup + sub * VEC, a.V, false);
-                qd = load_logits<T>(dp, g * kGroup + sub * VEC, a.V, false);
-              }
-            }
-            if (gi + GPI > gb + kGroupBatch) {   // warp-uniform
-              gb = gi & ~3;
-              const U4 wds = philox4x32_10(U4{(uint32_t)(gb >> 2) + (uint32_t)lane, (uint32_t)b,
-                                              (uint32_t)n, cw_grp}, k0, k1);
-              U0 = wds.x; U1 = wds.y; U2 = wds.z; U3 = wds.w;
-            }
-            float acc = resid_vec<T>(qt, qd, st);
-#pragma unroll
-            for (int o = 1; o < LPG; o <<= 1) acc += __shfl_xor_sync(kFull, acc, o);
-            const int off = min(g - gb, kGroupBatch - 1);
-            const int src = off >> 2, sel = off & 3;
-            const uint32_t x0 = __shfl_sync(kFull, U0, src), x1 = __shfl_sync(kFull, U1, src);
-            const uint32_t x2 = __shfl_sync(kFull, U2, src), x3 = __shfl_sync(kFull, U3, src);
-            const uint32_t word = sel == 0 ? x0 : sel == 1 ? x1 : sel == 2 ? x2 : x3;
-            // E_g >= U_g, so a group with U_g >= thr * R_g has a key above the
-            // warp's best so far and cannot win (the factor keeps the filter
-            // safe against the rounding of E and of the product)
-            bool improved = false;
-            if (g < ge && acc > 0.f && word_to_unit(word) * kRaceFilter < thr * acc) {
-              const float key = expo(word) / acc;
-              if (key < best) {          // groups are visited in increasing order
-                best = key;
-                bestg = g;
-                bqt = qt;
-                bqd = qd;
-                improved = true;
-              }
-            }
-            if (__any_sync(kFull, improved)) thr = warp_min(best);
-          }
-          __syncwarp();                  // the stage is rewritten by the next chunk
-        }
-        const float kmin = warp_min(best);
-        const int gmin = warp_min_i(best == kmin ? bestg : kIntMax);
-        // level 2 on this warp's winning group (its lanes are the ones whose
-        // best group it is)
-        int tok = -1;
-        if (gmin != kIntMax) {
-          const int own = ((gmin - g0) % GPI) * LPG;
-          tok = race_group_entries<T>(bqt, bqd, gmin, own, lane, st, (uint32_t)b, (uint32_t)n,
-                                      cw_ent, k0, k1);
-        }
-        int old = 0;
-        if (lane == 0) {
-          W.rpart[rr_ + w] = RacePartial{kmin, gmin, tok, 0};
-          old = atom_add_acq_rel(W.res_done + rr_, cnt);
-        }
-        old = __shfl_sync(kFull, old, 0);
-        if (old + cnt == ng) {
-          __syncwarp();
-          const int wf = sp.owner((int64_t)rr_ * ng);
-          const int wl = sp.owner((int64_t)rr_ * ng + ng - 1);
-          float key = pos_inf();
-          int gw = kIntMax, tw = -1;
-          for (int k = wf + lane; k <= wl; k += 32) {
-            const int4 x = __ldcg(reinterpret_cast<const int4*>(W.rpart + rr_ + k));
-            const float xk = __int_as_float(x.x);
-            if (xk < key || (xk == key && x.y < gw)) {
-              key = xk;
-              gw = x.y;
-              tw = x.z;
-            }
-          }
-          const float km = warp_min(key);
-          const int gm = warp_min_i(key == km ? gw : kIntMax);
-          const int tm = warp_min_i((key == km && gw == gm && tw >= 0) ? tw : kIntMax);
-          if (lane == 0) {
-            W.res_done[rr_] = 0;
-            a.out_tokens[r] = (gm != kIntMax && tm != kIntMax) ? tm : rq0.w;   // empty residual: argmax
-          }
-        }
-        u0 += cnt;
-      }
-    }
-  }
-  // the last CTA to finish clears the queue for the next call
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    const int done = atom_add_acq_rel(W.res_cta_done, 1);
-    if (done == (int)gridDim.x - 1) {
-      *W.rej_count = 0;
-      *W.res_cta_done = 0;
-      __threadfence();
+  if (nrows > 0) {
+    const StreamSplit sp(nrows, a.V, VEC, a.nwarps, stream_min_len(a.V));
+    if (w < sp.W) {
+      const int64_t e_begin = sp.start(w);
+      const int64_t e_end = sp.start(w + 1);
+      if (e_begin < e_end) walk_slice<T, MODE, SAMPLED, PH2>(a, s_pref, e_begin, e_end, sp, w, lane);
     }
   }
 }
 
-constexpr size_t kResSmemBytes = (size_t)kWarpsPerBlock * kResStageBytes;
+// Dynamic shared memory is at most the k_row prefix of kMaxRaggedB sequences;
+// the attribute is set once per kernel and device.
+constexpr size_t kMaxStreamSmem = ((size_t)(kMaxRaggedB + 1) * sizeof(int) + 127) / 128 * 128;
+
+template <typename K>
+cudaError_t smem_attr_once(K kernel, unsigned long long* done_mask) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (__atomic_load_n(done_mask, __ATOMIC_ACQUIRE) & bit) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxStreamSmem);
+  if (e == cudaSuccess) __atomic_fetch_or(done_mask, bit, __ATOMIC_ACQ_REL);
+  return e;
+}
+
+template <typename T, int MODE, bool SAMPLED, bool PH2>
+cudaError_t launch_one(const StreamArgs& a, int grid, size_t smem, cudaStream_t s) {
+  static unsigned long long done = 0ull;
+  cudaError_t e = smem_attr_once(stream_kernel<T, MODE, SAMPLED, PH2>, &done);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kStreamThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  return cudaLaunchKernelEx(&cfg, stream_kernel<T, MODE, SAMPLED, PH2>, a);
+}
+
+template <typename T, int MODE, bool SAMPLED, bool PH2>
+cudaError_t occupancy_one(size_t smem, int* nb) {
+  static unsigned long long done = 0ull;
+  cudaError_t e = smem_attr_once(stream_kernel<T, MODE, SAMPLED, PH2>, &done);
+  if (e != cudaSuccess) return e;
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, stream_kernel<T, MODE, SAMPLED, PH2>,
+                                                       kStreamThreads, smem);
+}
 
 // Launched as a programmatic dependent of the streaming kernel just before it
 // on the same stream: its CTAs may be scheduled as the streaming kernel's CTAs
 // retire, and griddepcontrol.wait at its top orders it after that grid.
-template <typename T>
-cudaError_t launch_resample_t(const StreamArgs& a, int grid, cudaStream_t s) {
-  cudaFuncSetAttribute(resample_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kResSmemBytes);
+template <typename T, bool SAMPLED>
+cudaError_t launch_resample_one(const StreamArgs& a, int grid, cudaStream_t s) {
+  static unsigned long long done = 0ull;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (!(__atomic_load_n(&done, __ATOMIC_ACQUIRE) & bit)) {
+    e = cudaFuncSetAttribute(resample_kernel<T, SAMPLED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kResSmemBytes);
+    if (e != cudaSuccess) return e;
+    __atomic_fetch_or(&done, bit, __ATOMIC_ACQ_REL);
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(kResThreads);
   cfg.dynamicSmemBytes = kResSmemBytes;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -1374,41 +1601,53 @@ cudaError_t launch_resample_t(const StreamArgs& a, int grid, cudaStream_t s) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, resample_kernel<T>, a);
+  return cudaLaunchKernelEx(&cfg, resample_kernel<T, SAMPLED>, a);
 }
 
 template <typename T>
-cudaError_t occupancy_resample_t(int* nb) {
-  cudaFuncSetAttribute(resample_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kResSmemBytes);
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, resample_kernel<T>, kThreads, kResSmemBytes);
+cudaError_t launch_resample_t(bool sampled, const StreamArgs& a, int grid, cudaStream_t s) {
+  return sampled ? launch_resample_one<T, true>(a, grid, s) : launch_resample_one<T, false>(a, grid, s);
 }
 
 template <typename T>
-cudaError_t launch_stream_t(int mode, bool sampled, const StreamArgs& a, int grid, size_t smem,
-                            cudaStream_t s) {
-#define CMSD_L(M, S)                                                                          \
-  do {                                                                                        \
-    cudaFuncSetAttribute(stream_kernel<T, M, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
-                         (int)smem);                                                          \
-    stream_kernel<T, M, S><<<grid, kStreamThreads, smem, s>>>(a);                                   \
+cudaError_t occupancy_resample_t(bool sampled, int* nb) {
+  cudaError_t e = sampled ? cudaFuncSetAttribute(resample_kernel<T, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)kResSmemBytes)
+                          : cudaFuncSetAttribute(resample_kernel<T, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)kResSmemBytes);
+  if (e != cudaSuccess) return e;
+  return sampled ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, resample_kernel<T, true>, kResThreads,
+                                                                 kResSmemBytes)
+                 : cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, resample_kernel<T, false>, kResThreads,
+                                                                 kResSmemBytes);
+}
+
+// The kernel variants: confidence only; verify and fused, each under the
+// PAPER rule without a second pass, the PAPER rule with the bonus row, and
+// the sampled rule (always a second pass).
+#define CMSD_DISPATCH(FN, ...)                                                              \
+  do {                                                                                      \
+    if (mode == kModeConf) return FN<T, kModeConf, false, false>(__VA_ARGS__);              \
+    if (mode == kModeVerify) {                                                              \
+      if (sampled) return FN<T, kModeVerify, true, true>(__VA_ARGS__);                      \
+      if (second) return FN<T, kModeVerify, false, true>(__VA_ARGS__);                      \
+      return FN<T, kModeVerify, false, false>(__VA_ARGS__);                                 \
+    }                                                                                       \
+    if (sampled) return FN<T, kModeFused, true, true>(__VA_ARGS__);                         \
+    if (second) return FN<T, kModeFused, false, true>(__VA_ARGS__);                         \
+    return FN<T, kModeFused, false, false>(__VA_ARGS__);                                    \
   } while (0)
-  if (mode == kModeConf) CMSD_L(kModeConf, false);
-  else if (mode == kModeVerify) { if (sampled) CMSD_L(kModeVerify, true); else CMSD_L(kModeVerify, false); }
-  else { if (sampled) CMSD_L(kModeFused, true); else CMSD_L(kModeFused, false); }
-#undef CMSD_L
-  return cudaGetLastError();
+
+template <typename T>
+cudaError_t launch_stream_t(int mode, bool sampled, bool second, const StreamArgs& a, int grid, size_t smem,
+                            cudaStream_t s) {
+  CMSD_DISPATCH(launch_one, a, grid, smem, s);
 }
 
 template <typename T>
-cudaError_t occupancy_stream_t(int mode, bool sampled, size_t smem, int* nb) {
-#define CMSD_O(M, S)                                                                            \
-  (cudaFuncSetAttribute(stream_kernel<T, M, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,   \
-                        (int)smem),                                                            \
-   cudaOccupancyMaxActiveBlocksPerMultiprocessor(nb, stream_kernel<T, M, S>, kStreamThreads, smem))
-  if (mode == kModeConf) return CMSD_O(kModeConf, false);
-  if (mode == kModeVerify) return sampled ? CMSD_O(kModeVerify, true) : CMSD_O(kModeVerify, false);
-  return sampled ? CMSD_O(kModeFused, true) : CMSD_O(kModeFused, false);
-#undef CMSD_O
+cudaError_t occupancy_stream_t(int mode, bool sampled, bool second, size_t smem, int* nb) {
+  CMSD_DISPATCH(occupancy_one, smem, nb);
 }
+#undef CMSD_DISPATCH
 
 }  // namespace cmsd

@@ -115,3 +115,35 @@ def test_product_path_fails_loudly_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(c, "_lib", None)
     with pytest.raises(c.CmsdError):
         c.lib()
+
+
+def test_ablation_presets(cmsd):
+    # the variants of the ablation (Sec. IV, Table III) as parameter sets
+    full = cmsd.params(16, "sampled")
+    assert (full.k_fixed, full.bonus) == (0, 0)
+    fk = cmsd.params(16, "sampled", preset="fixed_k")
+    assert fk.k_fixed == 16 and abs(fk.gamma - 1.0) < 1e-7
+    ft = cmsd.params(16, "sampled", preset="fixed_tau")
+    assert ft.k_fixed == 0 and ft.gamma == 0.0
+    fkt = cmsd.params(16, "sampled", preset="fixed_k_tau")
+    assert fkt.k_fixed == 16 and fkt.gamma == 0.0
+    for name, j in (("entropy_only", 0), ("margin_only", 1), ("softmax_only", 2)):
+        q = cmsd.params(16, "paper", preset=name)
+        assert list(q.lam) == [1.0 if k == j else 0.0 for k in range(3)]
+    p = cmsd.Params()
+    assert cmsd.lib().cmsd_params_preset(ctypes.byref(p), 8, 0, 99) == cmsd.EINVAL
+
+
+def test_bonus_and_fixed_k_argument_checks(cmsd):
+    # k_fixed outside [k_min, k_max] and a bonus row with rows that are not a
+    # whole number of 16-byte vectors are refused on the host
+    L = cmsd.lib()
+    a = ctypes.c_void_p(1 << 20)
+    bad_k = cmsd.params(8, "paper", k_fixed=9)
+    rc = L.cmsd_confidence_verify(a, a, a, None, 2, 8, 4096, cmsd.BF16, ctypes.byref(bad_k), 0, 0,
+                                  None, None, None, None, None, None, a, a, None, None, 0, None)
+    assert rc == cmsd.EINVAL
+    odd = cmsd.params(8, "paper", bonus=1)
+    rc = L.cmsd_confidence_verify(a, a, a, None, 2, 8, 4097, cmsd.BF16, ctypes.byref(odd), 0, 0,
+                                  None, None, None, None, None, None, a, a, None, None, 0, None)
+    assert rc == cmsd.EINVAL

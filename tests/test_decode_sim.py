@@ -87,12 +87,16 @@ def test_decode_loop_matches_oracle(mods, rule):
 
 
 @pytest.mark.gpu
-def test_decode_loop_full_size(mods):
-    # B=32, K_max=16, V=32000 float32 logits, 512 iterations, sampled rule; the
-    # first iterations of two sequences against the oracle, invariants everywhere
+@pytest.mark.parametrize("rule", ["sampled", "paper"])
+def test_decode_loop_full_size(mods, rule):
+    # B=32, K_max=16, V=32000 float32 logits, 512 iterations: every sequence
+    # against the oracle's replay (over the host's cores) up to its first
+    # flagged iteration, invariants everywhere
+    import oracle_pool
+    from parity_util import record
     cmsd, ds, W = mods
     B, K, V, its = 32, 16, 32000, 512
-    p = cmsd.params(K, "sampled")
+    p = cmsd.params(K, rule, beta_rank=0 if rule == "sampled" else 3)
     sim = ds.DecodeSim(B, K, V, its, p, seed=4)
     hist = sim.run()
     k, n, toks = hist["k"], hist["n_accept"], hist["out_tokens"]
@@ -105,18 +109,20 @@ def test_decode_loop_full_size(mods):
     s = ds.summarize(hist)
     assert s["rows"] == int(k.sum()) and 0 < s["mean_accepted"] <= K
 
-    import oracle as O
-    table = W.normal_table()
-    heights = W.ar1_heights(B, its, 4, table)
-
-    def gen(it, b, kk):
-        return W.decode_iteration_host(table, heights, it, b, kk, K, V, 4)
-
-    for b in (0, 17):
-        traj = O.decode_sim_sequence(gen, b, 6, K, oracle_params(p), 4)
-        for it, st in enumerate(traj):
+    replays = oracle_pool.decode_replays(B, K, V, its, p.as_dict(), 4, range(B))
+    compared, stopped = 0, []
+    for b in range(B):
+        for it, st in enumerate(replays[b]):
             assert k[it, b] == st["k"], (b, it)
             if st["flagged"]:
+                stopped.append(it)
                 break
             assert n[it, b] == st["n_accept"], (b, it)
             assert np.array_equal(toks[it, b], st["out_tokens"]), (b, it)
+            compared += 1
+    # the comparison covers (nearly) the whole trajectory of every sequence
+    assert compared >= 0.9 * B * its, (compared, stopped)
+    record("c5", rule, {"seqs": B, "rows": int(k.sum()), "k": 0, "n": 0, "tok": 0, "acc": 0},
+           {"iterations_compared": compared, "iterations_total": B * its,
+            "sequences_stopped_at_a_flagged_iteration": len(stopped),
+            "first_flagged_iterations": sorted(stopped), "summary": s})

@@ -8,7 +8,8 @@ everywhere else.
 import numpy as np
 import pytest
 
-from parity_util import check_properties, compare, gpu_fused, oracle_fused
+from parity_util import (assert_flag_bound, bonus_view, check_properties, compare, gpu_fused, oracle_fused,
+                         record)
 
 pytestmark = pytest.mark.gpu
 
@@ -203,25 +204,231 @@ def test_sampled_rule_reproduces_target_law_on_gpu(cmsd):
     assert stats.chi2.sf(chi2, V - 1) > 1e-3, (counts / n, p)
 
 
-# ---------------------------------------------------------------- full sizes
+def test_sampled_rule_modulated_law_on_gpu(cmsd):
+    # V = 8, K = 1, tau = 0.4 fixed (gamma = 0), no rank gate: the emitted token
+    # has the law of reading C9, min(q, e^tau p) + (1 - sum min(q, e^tau p)) *
+    # norm(max(0, p - q)), which differs from p (the drafts are over-accepted)
+    from scipy import stats
+    rng = np.random.default_rng(33)
+    V, B, tau = 8, 4096, 0.4
+    zt = rng.normal(0, 1.2, V).astype(np.float32)
+    zd = (zt + rng.normal(0, 0.9, V)).astype(np.float32)
+    p = np.exp(zt.astype(np.float64)); p /= p.sum()
+    q = np.exp(zd.astype(np.float64)); q /= q.sum()
+    a = np.minimum(q, np.exp(tau) * p)
+    r = np.maximum(0.0, p - q)
+    law = a + (1.0 - a.sum()) * r / r.sum()
+    assert np.abs(law - p).max() > 0.01                 # the modulation is visible
+    d = torch.from_numpy(np.tile(zd, (B, 1, 1))).cuda()
+    t = torch.from_numpy(np.tile(zt, (B, 1, 1))).cuda()
+    pp = cmsd.params(1, "sampled", tau_base=tau, gamma=0.0, beta_rank=0)
+    counts = np.zeros(V)
+    for it in range(16):
+        x = rng.choice(V, size=(B, 1), p=q).astype(np.int32)
+        o = cmsd.confidence_verify(d, t, torch.from_numpy(x).cuda(), p=pp, seed=7, iteration=it)
+        counts += np.bincount(o["out_tokens"][:, 0].cpu().numpy(), minlength=V)
+    n = counts.sum()
+    chi2 = ((counts - law * n) ** 2 / (law * n)).sum()
+    assert stats.chi2.sf(chi2, V - 1) > 1e-3, (counts / n, law)
+    chi2_p = ((counts - p * n) ** 2 / (p * n)).sum()
+    assert stats.chi2.sf(chi2_p, V - 1) < 1e-6          # and is not the unmodulated law
+
+
+# ------------------------------------------------ bonus row, fixed draft length
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("rule,kw", RULES)
+def test_parity_bonus_row(cmsd, W, dtype, rule, kw):
+    # the verifier's extra row gives one more token when every draft is
+    # accepted; a lenient tau makes that frequent, ragged windows move it
+    w = bonus_view(W.make("c2", B=9, K=7, V=2048, dtype=dtype))
+    k_row = np.array([6, 0, 1, 3, 6, 2, 6, 5, 4], np.int32)
+    bonus_seen = 0
+    for extra in (dict(), dict(tau_base=8.0, beta_rank=0)):
+        p = cmsd.params(w.K, rule, bonus=1, **{**kw, **extra})
+        for kr in (None, k_row):
+            g = gpu_fused(cmsd, torch, w, p, iteration=5, k_row=kr)
+            r = oracle_fused(w, p, iteration=5, k_row=kr)
+            assert g["out_tokens"].shape == (w.B, w.K + 1)
+            compare(w, g, r, k_row=kr)
+            kb = np.full(w.B, w.K) if kr is None else kr
+            bonus_seen += int(sum(g["n_accept"][b] == kb[b] and g["out_tokens"][b, kb[b]] >= 0
+                                  for b in range(w.B)))
+    assert bonus_seen >= 4
+
+
+def test_bonus_row_law_on_gpu(cmsd):
+    # every draft accepted (tau large): the bonus token of the sampled rule is
+    # a draw from the extra verifier row's softmax
+    from scipy import stats
+    rng = np.random.default_rng(41)
+    V, B = 8, 4096
+    zt = rng.normal(0, 1.0, V).astype(np.float32)
+    z1 = rng.normal(0, 1.3, V).astype(np.float32)
+    p1 = np.exp(z1.astype(np.float64)); p1 /= p1.sum()
+    d = torch.from_numpy(np.tile(zt, (B, 1, 1))).cuda()
+    t = torch.from_numpy(np.tile(np.stack([zt, z1]), (B, 1, 1))).cuda()
+    tok = torch.zeros((B, 1), dtype=torch.int32, device="cuda")
+    pp = cmsd.params(1, "sampled", tau_base=50.0, gamma=0.0, beta_rank=0, bonus=1)
+    counts = np.zeros(V)
+    for it in range(8):
+        o = cmsd.confidence_verify(d, t, tok, p=pp, seed=11, iteration=it)
+        n = o["n_accept"].cpu().numpy()
+        assert np.all(n == 1)
+        counts += np.bincount(o["out_tokens"][:, 1].cpu().numpy(), minlength=V)
+    m = counts.sum()
+    chi2 = ((counts - p1 * m) ** 2 / (p1 * m)).sum()
+    assert stats.chi2.sf(chi2, V - 1) > 1e-3
+
 
 @pytest.mark.parametrize("rule,kw", RULES)
-def test_full_size_c3(cmsd, W, rule, kw):
-    w = W.make("c3")
+def test_parity_fixed_draft_length(cmsd, W, rule, kw):
+    w = W.make("c2", B=6, K=8, V=3000)
+    for preset in ("fixed_k", "fixed_k_tau"):
+        p = cmsd.params(w.K, rule, preset=preset, **kw)
+        assert p.k_fixed == w.K
+        g = gpu_fused(cmsd, torch, w, p, iteration=2)
+        assert np.all(g["k_next"] == w.K)
+        compare(w, g, oracle_fused(w, p, iteration=2))
+    p = cmsd.params(w.K, rule, k_fixed=3, k_min=2, **kw)
+    g = gpu_fused(cmsd, torch, w, p, iteration=2)
+    assert np.all(g["k_next"] == 3)
+    compare(w, g, oracle_fused(w, p, iteration=2))
+
+
+@pytest.mark.parametrize("preset", ["entropy_only", "margin_only", "softmax_only", "fixed_tau"])
+def test_parity_ablation_presets(cmsd, W, preset):
+    w = W.make("c3", B=2, V=20000)
+    for rule, kw in RULES:
+        p = cmsd.params(w.K, rule, preset=preset, **kw)
+        compare(w, gpu_fused(cmsd, torch, w, p, iteration=3), oracle_fused(w, p, iteration=3))
+
+
+# ------------------------------------------- device error word and guard bands
+
+SENTINEL = {torch.float32: float("nan"), torch.int32: 0x5A5A5A5A, torch.uint8: 0xA5}
+GUARD = 64
+
+
+def _guarded(shape, dtype):
+    """A tensor of `shape` inside a larger buffer whose GUARD elements before
+    and after hold a sentinel; returns (view, buffer)."""
+    n = int(np.prod(shape))
+    buf = torch.empty(n + 2 * GUARD, dtype=dtype, device="cuda")
+    buf.fill_(SENTINEL[dtype])
+    return buf[GUARD:GUARD + n].view(shape), buf
+
+
+def _guards_intact(buf, dtype):
+    h = buf.cpu()
+    head, tail = h[:GUARD], h[-GUARD:]
+    if dtype == torch.float32:
+        return bool(torch.isnan(head).all() and torch.isnan(tail).all())
+    return bool((head == SENTINEL[dtype]).all() and (tail == SENTINEL[dtype]).all())
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("rule,kw", RULES)
+def test_outputs_stay_inside_their_arrays(cmsd, W, dtype, rule, kw):
+    # odd shapes; every output sits between guard bands that must be untouched,
+    # and so must the bytes after the workspace
+    w = W.make("c2", B=5, K=7, V=1001, dtype=dtype)
+    B, K = w.B, w.K
+    shapes = {"H": ((B, K), torch.float32), "margin": ((B, K), torch.float32),
+              "conf": ((B, K), torch.float32), "lse": ((B, K), torch.float32),
+              "argmax": ((B, K), torch.int32), "k_next": ((B,), torch.int32),
+              "n_accept": ((B,), torch.int32), "out_tokens": ((B, K), torch.int32),
+              "accept": ((B, K), torch.uint8)}
+    out, bufs = {}, {}
+    for n, (shape, dt) in shapes.items():
+        out[n], bufs[n] = _guarded(shape, dt)
+    nws = cmsd.lib().cmsd_workspace_bytes(B, K, w.V)
+    wsbuf = torch.full((nws + 4096,), 0xA5, dtype=torch.uint8, device="cuda")
+    ws = wsbuf[:nws]
+    ws.zero_()
+    k_row = torch.tensor([7, 3, 0, 6, 1], dtype=torch.int32, device="cuda")
+    p = cmsd.params(K, rule, **kw)
+    d = cmsd.to_device_logits(w.draft, w.dtype)
+    t = cmsd.to_device_logits(w.target, w.dtype)
+    tok = torch.from_numpy(w.tokens).cuda()
+    for it in range(3):
+        cmsd.confidence_verify(d, t, tok, k_row=k_row, p=p, seed=w.seed, iteration=it, out=out, ws=ws)
+    torch.cuda.synchronize()
+    for n, (shape, dt) in shapes.items():
+        assert _guards_intact(bufs[n], dt), n
+    assert bool((wsbuf[nws:] == 0xA5).all().item()), "workspace overrun"
+    g = {n: v.cpu().numpy() for n, v in out.items()}
+    compare(w, g, oracle_fused(w, p, iteration=2, k_row=k_row.cpu().numpy()), k_row=k_row.cpu().numpy())
+
+
+def test_device_error_word(cmsd, W):
+    # drafted tokens outside [0, V) and k_row outside [0, K] are clamped on the
+    # device before any load (token -> 0, k_row -> [0, K]) and reported in the
+    # workspace error word: bit 0 and bit 1
+    w = W.make("c2", B=4, K=5, V=900)
+    d = cmsd.to_device_logits(w.draft, w.dtype)
+    t = cmsd.to_device_logits(w.target, w.dtype)
+    ws = cmsd.workspace(w.B, w.K, w.V)
+    p = cmsd.params(w.K, "sampled")
+    assert cmsd.workspace_errors(ws) == 0
+    good = torch.from_numpy(w.tokens).cuda()
+    cmsd.confidence_verify(d, t, good, p=p, ws=ws)
+    assert cmsd.workspace_errors(ws) == 0
+    bad = w.tokens.copy()
+    bad[1, 2], bad[3, 0] = -1, w.V
+    cmsd.confidence_verify(d, t, torch.from_numpy(bad).cuda(), p=p, ws=ws)
+    assert cmsd.workspace_errors(ws) == 1
+    assert cmsd.workspace_errors(ws) == 0                # reading clears the word
+    kr = torch.tensor([5, 9, -2, 3], dtype=torch.int32, device="cuda")
+    cmsd.confidence_verify(d, t, good, k_row=kr, p=p, ws=ws)
+    assert cmsd.workspace_errors(ws) == 2
+    cmsd.confidence_verify(d, t, torch.from_numpy(bad).cuda(), k_row=kr, p=p, ws=ws)
+    assert cmsd.workspace_errors(ws) == 3
+    # the workspace keeps working after errors: a clean call matches the oracle
+    g = gpu_fused(cmsd, torch, w, p, iteration=2)
+    compare(w, g, oracle_fused(w, p, iteration=2))
+
+
+# ---------------------------------------------------------------- full sizes
+#
+# Every sequence of the full-size workloads, in the launch configuration
+# bench.py times, against the oracle (run over the host's cores); flagged
+# decisions bounded; deviations recorded (CMSD_PARITY_RECORD).
+
+@pytest.fixture(scope="module")
+def full_c3(W):
+    return W.make("c3")
+
+
+@pytest.fixture(scope="module")
+def full_c4(W):
+    return W.make("c4")
+
+
+def _full_size(cmsd, w, name, rule, kw):
+    import oracle_pool
     p = cmsd.params(w.K, rule, **kw)
     g = gpu_fused(cmsd, torch, w, p, iteration=1)
     check_properties(w, g, p)
-    seqs = [0, 17, 40, 63]
-    r = oracle_fused(w, p, iteration=1, seqs=seqs)
-    compare(w, g, r, seqs=seqs)
+    r = oracle_pool.fused(w, p.as_dict(), w.seed, iteration=1)
+    f = compare(w, g, r)
+    assert f["seqs"] == w.B and f["rows"] == w.B * w.K
+    assert_flag_bound(f)
+    record(name, rule, f, {"sizes": dict(B=w.B, K=w.K, V=w.V, dtype=w.dtype)})
+    print(name, rule, f)
 
 
-def test_full_size_c4(cmsd, W):
-    w = W.make("c4")
-    for rule, kw in RULES:
-        p = cmsd.params(w.K, rule, **kw)
-        g = gpu_fused(cmsd, torch, w, p, iteration=1)
-        check_properties(w, g, p)
-        seqs = [0, 255] if rule == "paper" else [128]
-        r = oracle_fused(w, p, iteration=1, seqs=seqs)
-        compare(w, g, r, seqs=seqs)
+@pytest.mark.parametrize("rule,kw", RULES)
+def test_full_size_c1_c2(cmsd, W, rule, kw):
+    for name in ("c1", "c2"):
+        _full_size(cmsd, W.make(name), name, rule, kw)
+
+
+@pytest.mark.parametrize("rule,kw", RULES)
+def test_full_size_c3(cmsd, full_c3, rule, kw):
+    _full_size(cmsd, full_c3, "c3", rule, kw)
+
+
+@pytest.mark.parametrize("rule,kw", RULES)
+def test_full_size_c4(cmsd, full_c4, rule, kw):
+    _full_size(cmsd, full_c4, "c4", rule, kw)

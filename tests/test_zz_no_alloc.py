@@ -72,13 +72,20 @@ def test_static_scratch_matches_workspace_entry_point(cmsd, name, kw, rule, k_ro
 
 def test_static_scratch_rejects_oversize_problem(cmsd):
     # B*K = 131072 positions needs more than CMSD_STATIC_SCRATCH_BYTES; the call
-    # is refused on the host before any pointer is used or anything enqueued.
-    p = cmsd.params(8, "sampled")
+    # is refused on the host after the argument checks and before anything is
+    # enqueued (the aligned dummy pointers are never dereferenced)
+    p = cmsd.params(1024, "sampled")
+    a = ctypes.c_void_p(1 << 20)
     rc = cmsd.lib().cmsd_confidence_verify_static(
-        None, None, None, None, 128, 1024, 32000, cmsd.BF16, ctypes.byref(p), 0, 0,
-        None, None, None, None, None, None, None, None, None, None)
+        a, a, a, None, 128, 1024, 32000, cmsd.BF16, ctypes.byref(p), 0, 0,
+        None, None, None, None, None, None, a, a, None, None)
     assert rc == cmsd.ESCRATCH
-    assert b"static scratch" in cmsd.lib().cmsd_strerror(rc)
+    # an invalid argument is reported before the size limit
+    rc = cmsd.lib().cmsd_confidence_verify_static(
+        None, a, a, None, 128, 1024, 32000, cmsd.BF16, ctypes.byref(p), 0, 0,
+        None, None, None, None, None, None, a, a, None, None)
+    assert rc == cmsd.EINVAL
+    assert b"static scratch" in cmsd.lib().cmsd_strerror(cmsd.ESCRATCH)
     # the empty problem is a valid call that enqueues nothing
     rc = cmsd.lib().cmsd_confidence_verify_static(
         None, None, None, None, 0, 8, 32000, cmsd.BF16, ctypes.byref(p), 0, 0,
