@@ -1,18 +1,22 @@
 #!/usr/bin/env python3
 """Benchmark of the fused CM-ASD logits pass (confidence + verification).
 
-Workload: recipe c3 -- B=64 sequences, K=8 drafted positions, V=128256,
-bfloat16 drafter and target logits (Zipf(1.1) profile x4 over a per-row
-permutation + 0.5 N(0,1); target = drafter + N(0,1); drafted tokens sampled
-from the drafter), SAMPLED rule (Philox acceptance + residual draw).
+Headline workload: recipe c3 -- B=64 sequences, K=8 drafted positions,
+V=128256, bfloat16 drafter and target logits (Zipf(1.1) profile x4 over a
+per-row permutation + 0.5 N(0,1); target = drafter + N(0,1); drafted tokens
+sampled from the drafter), SAMPLED rule (Philox acceptance + residual draw).
 
 A step is one call of cmsd_confidence_verify over one batch: the streaming
-kernel (every drafter and target logit read once) plus the residual-resample
-kernel over the rejected row pair of each sequence.  Two distinct input sets
+kernel (every drafter and target logit read once) plus the resample kernel
+over the rejected row pair of each sequence.  Two distinct input sets
 (2 x 263 MB, each larger than the 129 MB L2) alternate between steps.
 
-Prints one JSON line (rank 0).  --impl reference times the CPU oracle on a
-bounded sample of the same workload instead.
+Besides the headline, one JSON line carries (rank 0, one GPU): the other
+workloads (c1 latency, c2, c4, c3 under the paper's own rule), the decode-loop
+simulation (c5) with its generation and pass timed apart and the ablation
+variants of Table III, the CPU oracle timed on all host cores with a live
+parity check of its sample, and the flagged-decision counts of the full-size
+parity record.  --impl reference times the CPU oracle instead.
 """
 from __future__ import annotations
 
@@ -33,6 +37,8 @@ sys.path.insert(0, ROOT)
 WORKLOAD = "c3"
 METRIC = "confidence+verify logit rows/s at V=128256 (B=64, K=8, bf16 logits)"
 UNIT = "rows/s"
+C3_DESC = ("c3: B=64 K=8 V=128256 bf16 logits, Zipf(1.1)x4 profile over a per-row permutation + 0.5N(0,1); "
+           "target = drafter + N(0,1); drafted ~ softmax")
 
 
 def log(*a):
@@ -60,18 +66,38 @@ def kernel_sources_sha():
     return h.hexdigest()[:16]
 
 
-def ncu_traffic():
+def ncu_traffic(workload, rule):
     """Per-launch DRAM bytes of the streaming kernel from the committed ncu
-    summary; None when the kernel sources changed since it was captured."""
+    summary for this workload and rule; None when the kernel sources changed
+    since it was captured."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
-            d = json.load(f)
-        if d.get("sources_sha256_16") != kernel_sources_sha():
-            return None
-        return d
+            recs = json.load(f)
+        recs = recs if isinstance(recs, list) else [recs]
+        for d in recs:
+            if d.get("workload") == workload and d.get("rule") == rule and \
+                    d.get("sources_sha256_16") == kernel_sources_sha():
+                return d.get("bytes_per_launch")
     except Exception:
-        return None
+        pass
+    return None
+
+
+def parity_record(workload, rule):
+    """Flagged decisions and largest deviations of the full-size parity test
+    (profiles/parity_full_size.json, written from the GPU tests' records)."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "parity_full_size.json")) as f:
+            d = json.load(f)
+        for r in d.get("records", []):
+            if r.get("workload") == workload and r.get("rule") == rule:
+                out = {k: r[k] for k in ("sequences", "decisions", "flagged", "max_abs_err") if k in r}
+                out["current_kernels"] = d.get("sources_sha256_16") == kernel_sources_sha()
+                return out
+    except Exception:
+        pass
+    return None
 
 
 class ClockSampler:
@@ -149,69 +175,295 @@ def job_rows_per_s(world, rows_per_rank, steps, ms_total):
     return world * rows_per_rank * steps / (ms_total * 1e-3)
 
 
-def oracle_rows_per_s(w, p_dict, budget_s, seeds_from=0, max_rows=None):
-    """Time the CPU oracle on whole sequences of w until budget_s is used."""
-    import oracle as O
-    d64 = O.logits_to_f64(w.draft[seeds_from:seeds_from + 1], w.dtype)
-    t64 = O.logits_to_f64(w.target[seeds_from:seeds_from + 1], w.dtype)
-    P = O.Params(**p_dict)
-    rows = 0
-    t0 = time.perf_counter()
-    b = 0
-    while True:
-        O.confidence_verify(d64, t64, w.tokens[seeds_from:seeds_from + 1], P, seed=w.seed, iteration=b)
-        rows += w.K
-        b += 1
-        if time.perf_counter() - t0 >= budget_s or (max_rows and rows >= max_rows):
-            break
-    dt = time.perf_counter() - t0
-    return rows / dt, rows, dt
+def stats_ms(xs):
+    xs = sorted(xs)
+    return {"median": statistics.median(xs), "p10": float(np.percentile(xs, 10)),
+            "p90": float(np.percentile(xs, 90)), "min": xs[0], "max": xs[-1], "n": len(xs)}
 
+
+def time_total(torch, calls, nsteps, it0=0):
+    """Two CUDA events around nsteps steps on the launching stream: total ms."""
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for i in range(nsteps):
+        calls[i % len(calls)](iteration=it0 + i)
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1)
+
+
+def time_steps(torch, calls, nsteps, it0=0):
+    """CUDA events around every step on the launching stream: (total ms, per-step ms).
+    An event between steps costs about 2 us of device time per step on this
+    path, so the spread comes from this pass and throughput from time_total."""
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(nsteps + 1)]
+    ev[0].record()
+    for i in range(nsteps):
+        calls[i % len(calls)](iteration=it0 + i)
+        ev[i + 1].record()
+    torch.cuda.synchronize()
+    return ev[0].elapsed_time(ev[-1]), [ev[i].elapsed_time(ev[i + 1]) for i in range(nsteps)]
+
+
+def kernel_times(cmsd, torch, calls, nsteps):
+    """The library's per-kernel events (streaming, resample) over nsteps calls."""
+    cmsd.profile_start(nsteps)
+    for i in range(nsteps):
+        calls[i % len(calls)](iteration=i)
+    torch.cuda.synchronize()
+    return cmsd.profile_stop(nsteps)
+
+
+# ---------------------------------------------------------------- CPU oracle
+
+def _oracle_seq_task(task):
+    """Oracle over whole sequences (worker process): returns rows, seconds and
+    the per-sequence results used by the live parity check."""
+    draft, target, tokens, dtype, pdict, seed, iteration, b_index = task
+    import oracle as O
+    P = O.Params(**pdict)
+    t0 = time.perf_counter()
+    res = []
+    for j, b in enumerate(b_index):
+        d = O.logits_to_f64(draft[j:j + 1], dtype)
+        t = O.logits_to_f64(target[j:j + 1], dtype)
+        r = O.confidence(d, P)
+        v = O.verify_sequence(d[0], t[0], tokens[j], r.conf[0], d.shape[1], P, seed, int(b), iteration)
+        res.append({"b": int(b), "k_next": int(r.k_next[0]), "k_flag": bool(r.k_flag[0]),
+                    "n_accept": int(v["n_accept"]), "n_flag": bool(v["n_flag"]),
+                    "out_tokens": v["out_tokens"].tolist(), "tok_flag": bool(v["tok_flag"]),
+                    "conf": r.conf[0].tolist()})
+    return len(b_index) * draft.shape[1], time.perf_counter() - t0, res
+
+
+def _seq_task(w, b, pdict, seed, iteration):
+    return (np.ascontiguousarray(w.draft[b:b + 1]), np.ascontiguousarray(w.target[b:b + 1]),
+            np.ascontiguousarray(w.tokens[b:b + 1]), w.dtype, pdict, seed, iteration, [b])
+
+
+def oracle_pool_run(w, pdict, seed, iteration, budget_s, procs):
+    """Time the oracle on whole sequences of w over `procs` worker processes
+    (spawned, so no worker is a fork of this CUDA process) for about
+    budget_s; returns (rows/s, rows, seconds, per-sequence results)."""
+    import multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(procs) as pool:
+        pool.map(_oracle_seq_task, [_seq_task(w, 0, pdict, seed, iteration)] * procs)   # workers warm
+        t0 = time.perf_counter()
+        out = pool.map(_oracle_seq_task, [_seq_task(w, b % w.B, pdict, seed, iteration) for b in range(procs)])
+        t_round = time.perf_counter() - t0
+        rounds = max(0, int((budget_s - t_round) / max(t_round, 1e-3)))
+        more = [_seq_task(w, (procs + j) % w.B, pdict, seed, iteration) for j in range(rounds * procs)]
+        out += pool.map(_oracle_seq_task, more)
+        dt = time.perf_counter() - t0
+    rows = sum(x[0] for x in out)
+    seen, results = set(), []
+    for x in out:
+        for r in x[2]:
+            if r["b"] not in seen:
+                seen.add(r["b"])
+                results.append(r)
+    return rows / dt, rows, dt, results
+
+
+def live_parity(results, g, K):
+    """Compare the oracle's per-sequence results with the GPU's outputs:
+    flagged decisions and mismatches (outside the flagged ones)."""
+    flagged = mism = 0
+    maxc = 0.0
+    for r in results:
+        b = r["b"]
+        maxc = max(maxc, float(np.max(np.abs(g["conf"][b].astype(np.float64) - np.array(r["conf"])))))
+        if r["k_flag"]:
+            flagged += 1
+        elif g["k_next"][b] != r["k_next"]:
+            mism += 1
+        if r["n_flag"]:
+            flagged += 1
+        elif g["n_accept"][b] != r["n_accept"]:
+            mism += 1
+        if r["tok_flag"]:
+            flagged += 1
+        elif list(g["out_tokens"][b]) != r["out_tokens"]:
+            mism += 1
+    return {"sequences": len(results), "decisions": 3 * len(results), "flagged": flagged,
+            "mismatches": mism, "max_abs_err_conf": maxc}
+
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:   # pragma: no cover
+        return os.cpu_count() or 1
+
+
+# ---------------------------------------------------------------- reference arm
 
 def run_reference(args):
-    """CPU oracle as the reference arm (rank 0 only)."""
+    """CPU oracle as the reference arm (rank 0 only), on all host cores."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
     os.environ.setdefault("OMP_NUM_THREADS", "1")
-    import oracle as O
     from paper_2508_15371_gb300 import workloads as W
-    w = W.make(WORKLOAD, B=1)
-    P = O.Params(k_min=1, k_max=w.K, rule="sampled", beta_rank=0,
-                 lam=tuple(float(np.float32(1 / 3)) for _ in range(3)),
-                 tau_base=float(np.float32(0.1)))
-    d64 = O.logits_to_f64(w.draft, w.dtype)
-    t64 = O.logits_to_f64(w.target, w.dtype)
-    # calibrate one sequence, then size the per-step sample so the run ends in ~2 minutes
-    t0 = time.perf_counter()
-    O.confidence_verify(d64, t64, w.tokens, P, seed=w.seed, iteration=0)
-    t_seq = time.perf_counter() - t0
+    w = W.make(WORKLOAD, B=16)
+    pdict = dict(k_min=1, k_max=w.K, rule="sampled", beta_rank=0,
+                 lam=tuple(float(np.float32(1 / 3)) for _ in range(3)), tau_base=float(np.float32(0.1)))
+    procs = max(1, min(16, host_cores()))
+    # each step: one whole sequence per worker, timed as a batch
     total = args.steps + args.warmup
-    rows_per_step = w.K
-    if total * t_seq > 120.0:
-        rows_per_step = max(1, int(120.0 / total / (t_seq / w.K)))
-    k_row = None if rows_per_step >= w.K else np.array([rows_per_step], np.int64)
-    for it in range(args.warmup):
-        O.confidence_verify(d64, t64, w.tokens, P, seed=w.seed, iteration=it, k_row=k_row)
-    t0 = time.perf_counter()
-    for it in range(args.steps):
-        O.confidence_verify(d64, t64, w.tokens, P, seed=w.seed, iteration=it, k_row=k_row)
-    dt = time.perf_counter() - t0
-    rows = args.steps * min(rows_per_step, w.K)
+    times = []
+    import multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(procs) as pool:
+        for st in range(total):
+            tasks = [_seq_task(w, (st * procs + j) % w.B, pdict, w.seed, st) for j in range(procs)]
+            t0 = time.perf_counter()
+            pool.map(_oracle_seq_task, tasks)
+            dt = time.perf_counter() - t0
+            if st >= args.warmup:
+                times.append(dt)
+            if sum(times) > 150.0:
+                break
+    rows = len(times) * procs * w.K
+    dt = sum(times)
     value = rows / dt
-    sample = (f"{min(rows_per_step, w.K)} drafted positions (one sequence) of the B=64 K=8 V=128256 "
-              f"bf16 workload per step, float64 numpy oracle")
+    sample = (f"{procs} whole sequences (K={w.K} positions each, one per worker) of the B=64 K=8 V=128256 bf16 "
+              f"workload per step, float64 numpy oracle, {len(times)} steps")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "steps": len(times), "warmup": args.warmup, "ms_per_step": 1e3 * dt / len(times),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic",
-            "config": {"workload": "c3: B=64 K=8 V=128256 bf16 Zipf(1.1)x4 + 0.5N, target +N, drafted ~ softmax",
-                       "rule": "sampled", "sample_rows_per_step": min(rows_per_step, w.K)},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "config": {"workload": C3_DESC, "rule": "sampled", "sample_rows_per_step": procs * w.K},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": procs, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
 
+
+# ---------------------------------------------------------------- other workloads
+
+def bench_workload(cmsd, torch, dev, name, rule, steps, peak, nsets=1, graph_latency=False, **size):
+    """Device-resident timing of one workload: per-step times (median and
+    spread), the streaming kernel's time and its HBM roofline."""
+    from paper_2508_15371_gb300 import workloads as W
+    base = W.FULL_SIZES[name]["seed"]
+    sets = [W.make(name, seed=base + 100 * j, **size) for j in range(nsets)]
+    w0 = sets[0]
+    p = cmsd.params(w0.K, rule)
+    ws = cmsd.workspace(w0.B, w0.K, w0.V)
+    out = {"k_next": torch.empty(w0.B, dtype=torch.int32, device=dev),
+           "n_accept": torch.empty(w0.B, dtype=torch.int32, device=dev),
+           "out_tokens": torch.empty((w0.B, w0.K), dtype=torch.int32, device=dev)}
+    calls = []
+    for w in sets:
+        d = cmsd.to_device_logits(w.draft, w.dtype, dev)
+        t = cmsd.to_device_logits(w.target, w.dtype, dev)
+        tk = torch.from_numpy(w.tokens).to(dev)
+        calls.append(cmsd.FusedCall(d, t, tk, p, seed=w.seed, out=out, ws=ws))
+    desc = f"{name}: B={w0.B} K={w0.K} V={w0.V} {w0.dtype}"
+    K, V, rows, alg = w0.K, w0.V, w0.rows, w0.logit_bytes
+    es = 4 if w0.dtype == "f32" else 2
+    del sets, w0
+    for i in range(5):
+        calls[i % len(calls)](iteration=i)
+    torch.cuda.synchronize()
+    total = time_total(torch, calls, steps)
+    _, per = time_steps(torch, calls, steps)
+    k_ms, r_ms = kernel_times(cmsd, torch, calls, steps)
+    n = out["n_accept"].cpu().numpy()
+    rejected = int((n < K).sum()) if rule == "sampled" else 0
+    st = stats_ms(per)
+    km = statistics.median(k_ms)
+    res = {"workload": desc, "rule": rule,
+           "rows_per_s": rows * steps / (total * 1e-3), "ms_per_step": total / steps, "step_ms": st,
+           "kernel_ms": km, "resample_ms": statistics.median(r_ms) if rule == "sampled" else 0.0,
+           "algorithmic_bytes": alg, "kernel_gbs": alg / (km * 1e-3) / 1e9,
+           "kernel_frac": alg / (km * 1e-3) / 1e9 / peak,
+           "step_gbs": (alg + rejected * 2 * V * es) / (total / steps * 1e-3) / 1e9,
+           "l2": "inputs larger than L2" if alg > 129e6 else "L2-resident (inputs smaller than L2)",
+           "traffic": ncu_traffic(name, rule), "parity": parity_record(name, rule)}
+    res["step_frac"] = res["step_gbs"] / peak
+    if graph_latency:
+        # launch cost removed: the same call captured 20 times in a CUDA graph
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for i in range(20):
+                calls[0](iteration=i)
+        g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(10):
+            g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        res["latency_us_graph"] = e0.elapsed_time(e1) / 200 * 1e3
+        res["latency_us_launch"] = st["median"] * 1e3
+    del calls
+    torch.cuda.empty_cache()
+    return res
+
+
+def decode_sim_report(cmsd, torch, B=32, K=16, V=32000, iterations=512):
+    """Algorithm 1 as a decode loop over device-generated f32 logits (k_next
+    of each iteration is the next iteration's k_row), captured in a CUDA
+    graph: the whole loop, generation alone, and the pass alone timed with
+    CUDA events; then the ablation variants of Table III and the bonus row."""
+    from paper_2508_15371_gb300 import decode_sim
+
+    def one(preset="full", bonus=0, timing=False):
+        p = cmsd.params(K, "sampled", preset=preset, bonus=bonus)
+        sim = decode_sim.DecodeSim(B, K, V, iterations, p, seed=4)
+        sim.step(0)                      # first launches outside the capture
+        torch.cuda.synchronize()
+        g = sim.capture()
+        g.replay()
+        torch.cuda.synchronize()
+        hist = sim.history()
+        s = decode_sim.summarize(hist, bonus=bool(bonus))
+        if timing:
+            gg = sim.capture(generate=True, verify=False)
+            gv = sim.capture(generate=False, verify=True)
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+            e[0].record()
+            g.replay()
+            e[1].record()
+            gg.replay()
+            e[2].record()
+            gg.replay()
+            e[3].record()
+            gv.replay()
+            e[4].record()
+            gv.replay()
+            e[5].record()
+            torch.cuda.synchronize()
+            ms, ms_gen, ms_pass = e[0].elapsed_time(e[1]), e[2].elapsed_time(e[3]), e[4].elapsed_time(e[5])
+            hb = decode_sim.pass_bytes(hist, V, 4, bonus=bool(bonus))
+            s.update({"ms_per_iteration": ms / iterations, "rows_per_s": s["rows"] / (ms * 1e-3),
+                      "generation_ms_per_iteration": ms_gen / iterations,
+                      "pass_ms_per_iteration": ms_pass / iterations,
+                      "pass_rows_per_s": s["rows"] / (ms_pass * 1e-3),
+                      "pass_bytes_per_iteration": hb / iterations,
+                      "pass_gbs": hb / (ms_pass * 1e-3) / 1e9,
+                      "timing": "CUDA graph of the 512 iterations; generation and pass also captured and "
+                                "replayed alone (the pass over the last iteration's logits with the recorded "
+                                "windows), CUDA events"})
+        return s
+
+    rep = one(timing=True)
+    rep["workload"] = f"B={B} K_max={K} V={V} f32, {iterations} iterations, sampled rule, AR(1) spike heights"
+    rep["ablation"] = {}
+    keys = ("mean_k", "mean_accepted", "tokens_per_iteration", "rollbacks")
+    for preset in ("full", "fixed_k", "fixed_tau", "fixed_k_tau", "entropy_only", "margin_only", "softmax_only"):
+        s = one(preset)
+        rep["ablation"][preset] = {k: s[k] for k in keys}
+    s = one("full", bonus=1)
+    rep["ablation"]["full+bonus_row"] = {k: s[k] for k in keys}
+    return rep
+
+
+# ---------------------------------------------------------------- our arm
 
 def run_ours(args):
     import torch
@@ -229,6 +481,7 @@ def run_ours(args):
     else:
         torch.cuda.set_device(0)
     dev = torch.device("cuda", torch.cuda.current_device())
+    peak, peak_src = peaks()
 
     # ---- inputs (host generation, then resident in HBM) ---------------------
     t_gen = time.perf_counter()
@@ -252,7 +505,6 @@ def run_ours(args):
     launches_per_step = 2 if sampled else 1
 
     # ---- warm-up, clock sampler --------------------------------------------
-    uuid = None
     try:
         uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
     except Exception:   # noqa: BLE001
@@ -271,32 +523,25 @@ def run_ours(args):
             torch.cuda.synchronize()
     torch.cuda.synchronize()
 
-    # ---- timed region: device-resident inputs -----------------------------
+    # ---- timed region: device-resident inputs, two events ------------------
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
-    ev0 = torch.cuda.Event(enable_timing=True)
-    ev1 = torch.cuda.Event(enable_timing=True)
     t_wall0 = time.time()
-    ev0.record()
-    for it in range(args.steps):
-        calls[it % len(calls)](iteration=it)
-    ev1.record()
-    torch.cuda.synchronize()
+    ms_total = time_total(torch, calls, args.steps)
     t_wall1 = time.time()
     if dist:
         dist.barrier()
-    ms_total = ev0.elapsed_time(ev1)
+    # the same steps with an event after each: the spread of step times
+    _, per_step = time_steps(torch, calls, args.steps)
     clocks.stop()
     clk = clocks.summary(t_wall0, t_wall1)
-    # the same steps again with the library's per-kernel CUDA events (an event
+    # the same steps again with the library's per-kernel events (an event
     # between the two kernels serialises them, so this pass is not the one
     # `value` comes from): durations of the streaming and resample kernels
-    cmsd.profile_start(args.steps)
-    for it in range(args.steps):
-        calls[it % len(calls)](iteration=it)
-    torch.cuda.synchronize()
-    k_ms, r_ms = cmsd.profile_stop(args.steps)
+    k_ms, r_ms = kernel_times(cmsd, torch, calls, args.steps)
+    n_last = out["n_accept"].cpu().numpy()
+    rejected = int((n_last < K).sum()) if sampled else 0
     ms_total = max_over_ranks(ms_total, dist, dev)
     ms_step = ms_total / args.steps
     value = job_rows_per_s(world, rows, args.steps, ms_total)
@@ -339,93 +584,87 @@ def run_ours(args):
         e2e_step(j)
     e1.record()
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    e2e_ms = max_over_ranks(e2e_ms, dist, dev)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), dist, dev)
     e2e_value = job_rows_per_s(world, rows, e2e_steps, e2e_ms)
+    del host, dbuf
 
-    # ---- roofline of the streaming kernel ----------------------------------
-    peak, peak_src = peaks()
-    k_mean = statistics.mean(k_ms) if k_ms else float("nan")
-    r_mean = statistics.mean(r_ms) if r_ms else 0.0
-    achieved = alg_bytes / (k_mean * 1e-3) / 1e9
-    tr = ncu_traffic()
-    traffic = tr.get("bytes_per_launch") if tr and tr.get("workload") == WORKLOAD and tr.get("rule") == args.rule else None
+    # ---- roofline: the streaming kernel, and the whole step -----------------
+    k_med = statistics.median(k_ms)
+    achieved = alg_bytes / (k_med * 1e-3) / 1e9
+    step_stats = stats_ms(per_step)
+    resample_bytes = rejected * 2 * V * 2
+    step_gbs = (alg_bytes + resample_bytes) / (ms_step * 1e-3) / 1e9
 
     if rank != 0:
         if dist:
             dist.destroy_process_group()
         return 0
 
-    # ---- decode-loop simulation (rank 0, N = 1 only) -------------------------
-    dsim = None
-    if world == 1 and not args.no_decode_sim:
-        dsim = decode_sim_report()
+    extra = {}
+    if world == 1 and not args.no_extra:
+        # ---- the other workloads ---------------------------------------------
+        extra["workloads"] = [
+            bench_workload(cmsd, torch, dev, "c1", "sampled", 200, peak, graph_latency=True),
+            bench_workload(cmsd, torch, dev, "c1", "paper", 200, peak, graph_latency=True),
+            bench_workload(cmsd, torch, dev, "c2", "sampled", 200, peak),
+            bench_workload(cmsd, torch, dev, "c3", "paper", 200, peak, nsets=2),
+            bench_workload(cmsd, torch, dev, "c4", "sampled", 50, peak),
+            bench_workload(cmsd, torch, dev, "c4", "paper", 50, peak),
+        ]
+        # ---- decode-loop simulation --------------------------------------------
+        if not args.no_decode_sim:
+            extra["decode_sim"] = decode_sim_report(cmsd, torch)
 
-    # ---- CPU oracle baseline (rank 0, N = 1 only) ---------------------------
+    # ---- CPU oracle baseline, with a live parity check of its sample ---------
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        v, nrows, dt = oracle_rows_per_s(w0, p.as_dict(), budget_s=args.cpu_budget)
-        cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": f"{nrows} drafted positions ({nrows // K} sequence passes) of this workload, "
-                         f"float64 numpy, single thread, {dt:.1f} s"}
+        it_live = 777
+        gout = cmsd.confidence_verify(dsets[0][0], dsets[0][1], dsets[0][2], p=p, seed=w0.seed,
+                                      iteration=it_live, signals=True)
+        torch.cuda.synchronize()
+        g = {k2: v2.cpu().numpy() for k2, v2 in gout.items() if v2 is not None}
+        procs = max(1, min(16, host_cores()))
+        v, nrows, dt, results = oracle_pool_run(w0, p.as_dict(), w0.seed, it_live, args.cpu_budget, procs)
+        cpu = {"value": v, "unit": UNIT, "cores": procs, "kind": "oracle",
+               "sample": f"{nrows} drafted positions ({nrows // K} whole sequences) of this workload, float64 "
+                         f"numpy, {procs} worker processes (one per core), {dt:.1f} s"}
+        extra["live_parity"] = live_parity(results, g, K)
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": "c3: B=64 K=8 V=128256 bf16 logits, Zipf(1.1)x4 profile over a per-row "
-                               "permutation + 0.5N(0,1); target = drafter + N(0,1); drafted ~ softmax",
-                   "rule": args.rule, "logits": "bf16", "accumulate": "f32",
+        "config": {"workload": C3_DESC, "rule": args.rule, "logits": "bf16", "accumulate": "f32",
                    "l2": "inputs larger than L2: 2 alternating input sets of 263 MB each (L2 129 MB)",
                    "parallelism": f"dp{world} (independent batches per GPU)" if world > 1 else "single GPU"},
+        "step_ms": step_stats,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": traffic,
+                     "frac": achieved / peak, "traffic": ncu_traffic(WORKLOAD, args.rule),
                      "kernel": "stream_kernel (fused confidence + verify pass)",
-                     "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback 6800 GB/s",
-                     "algorithmic_bytes_per_launch": alg_bytes, "kernel_ms": k_mean,
-                     "kernel_timing": "CUDA events around each streaming-kernel launch, averaged over a "
-                                      "second pass of the same steps"},
-        "hbm_gbs_step": alg_bytes / (ms_step * 1e-3) / 1e9,
-        "resample_ms": r_mean,
+                     "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+                     else "fallback 6800 GB/s",
+                     "algorithmic_bytes_per_launch": alg_bytes, "kernel_ms": k_med,
+                     "kernel_timing": "CUDA events around each streaming-kernel launch (median over a second "
+                                      "pass of the same steps)"},
+        "step_roofline": {"achieved": step_gbs, "frac": step_gbs / peak, "unit": "GB/s",
+                          "bytes_per_step": alg_bytes + resample_bytes,
+                          "resample_bytes_per_step": resample_bytes,
+                          "note": "every logit once plus the rejected row pairs again, over the median step"},
+        "resample_ms": statistics.median(r_ms) if sampled else 0.0,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": e2e_steps},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk,
+        "parity": parity_record(WORKLOAD, args.rule),
+        "outputs_written": "n_accept, out_tokens, k_next (the per-position signals H, margin, argmax, conf, "
+                           "lse and the accept bits are not requested in the timed steps)",
     }
-    if dsim is not None:
-        line["decode_sim"] = dsim
+    line.update(extra)
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
     return 0
-
-
-def decode_sim_report(B=32, K=16, V=32000, iterations=512):
-    """Algorithm 1 as a decode loop over device-generated f32 logits: k_next of
-    each iteration is the next iteration's k_row.  Timed with CUDA events over
-    all iterations (logit generation included)."""
-    import torch
-    from paper_2508_15371_gb300 import cmsd, decode_sim
-    p = cmsd.params(K, "sampled")
-    sim = decode_sim.DecodeSim(B, K, V, iterations, p, seed=4)
-    for it in range(3):
-        sim.step(it)
-    torch.cuda.synchronize()
-    sim = decode_sim.DecodeSim(B, K, V, iterations, p, seed=4)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for it in range(iterations):
-        sim.step(it)
-    e1.record()
-    torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
-    hist = {"k": sim.hist_k.cpu().numpy(), "n_accept": sim.hist_n.cpu().numpy()}
-    s = decode_sim.summarize(hist)
-    s.update({"workload": f"B={B} K_max={K} V={V} f32, {iterations} iterations, sampled rule, AR(1) spike heights",
-              "ms_per_iteration": ms / iterations, "rows_per_s": s["rows"] / (ms * 1e-3),
-              "timing": "CUDA events over the loop, device logit generation included"})
-    return s
 
 
 def main():
@@ -435,9 +674,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--rule", choices=["sampled", "paper"], default="sampled")
-    ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-decode-sim", action="store_true", help="skip the decode-loop simulation report")
+    ap.add_argument("--no-extra", action="store_true", help="headline only (no other workloads, no decode loop)")
     ap.add_argument("--load-window", type=float, default=0.8,
                     help="seconds of untimed steps just before the timed region (clock sampling)")
     args = ap.parse_args()

@@ -8,7 +8,7 @@
  * paper_2508_15371_gb300/workloads.py (decode_row_host).  It stands in for the
  * paper's drafter and verifier models (Sec. IV.A), which are not available.
  *
- * Row (b, i), i < k_row[b], at iteration `it` (row id r = b * K_max + i):
+ * Row (b, i) at iteration `it` (row id r = b * (K_max + 1) + i):
  *   n1[v], n2[v] = table[u16] with u16 the 16-bit half (v & 1) of Philox4x32-10
  *                  word (v >> 1) & 3 of counter (v >> 3, r, it, 0xC0000002 / 0xC0000003),
  *                  key (seed lo, seed hi)
@@ -16,7 +16,9 @@
  *   draft[v]     = n1[v], plus heights_it[b] at the spike token (float add)
  *   target[v]    = draft[v] + 0.8f * n2[v]  (float multiply, then add)
  *   token[r]     = first argmax of draft
- * Rows with i >= k_row[b] are not written.
+ * Drafter rows and tokens are written for i < k_row[b]; verifier rows for
+ * i < k_row[b] + (Kt - K_max), i.e. with Kt = K_max + 1 also the row after the
+ * drafted window (the verifier's extra row).  Other rows are not written.
  */
 #ifndef CMSD_WORKLOAD_H
 #define CMSD_WORKLOAD_H
@@ -28,11 +30,13 @@ extern "C" {
 
 /* table: float[65536] device (normal quantiles); heights_it: float[B] device
  * (spike heights of this iteration); k_row: int32[B] device (NULL = K_max);
- * draft, target: float [B][K_max][V] device; tokens: int32 [B][K_max] device.
+ * Kt: verifier rows per sequence, K_max or K_max + 1;
+ * draft: float [B][K_max][V] device; target: float [B][Kt][V] device;
+ * tokens: int32 [B][K_max] device.
  * Returns 0, or -1 on a bad argument, -3 on a CUDA launch error. */
 int cmsd_gen_decode_rows(const float* table, const float* heights_it, uint32_t it, int B, int K_max,
-                         int V, const int32_t* k_row, uint64_t seed, float* draft, float* target,
-                         int32_t* tokens, void* stream);
+                         int Kt, int V, const int32_t* k_row, uint64_t seed, float* draft,
+                         float* target, int32_t* tokens, void* stream);
 
 #ifdef __cplusplus
 }

@@ -20,25 +20,28 @@ __device__ __forceinline__ uint32_t half16(const cmsd::U4& w, int j) {
   return (j & 1) ? (word >> 16) : (word & 0xFFFFu);
 }
 
+// One CTA per (b, i) slot of the [B][Kt] verifier layout.
 __global__ void __launch_bounds__(kThreads) gen_rows_kernel(const float* __restrict__ table,
                                                             const float* __restrict__ heights_it,
-                                                            uint32_t it, int B, int K_max, int V,
+                                                            uint32_t it, int B, int K_max, int Kt, int V,
                                                             const int32_t* __restrict__ k_row,
                                                             uint32_t k0, uint32_t k1, float* draft,
                                                             float* target, int32_t* tokens) {
-  const int row = blockIdx.x;
-  const int b = row / K_max;
-  const int i = row - b * K_max;
+  const int b = blockIdx.x / Kt;
+  const int i = blockIdx.x - b * Kt;
+  int k = K_max;
   if (k_row) {
-    int k = k_row[b];
+    k = k_row[b];
     k = k < 0 ? 0 : (k > K_max ? K_max : k);
-    if (i >= k) return;
   }
+  const bool has_draft = i < k;
+  if (!has_draft && i >= k + (Kt - K_max)) return;
+  const int row = b * (K_max + 1) + i;          // generator row id
   const float h = heights_it[b];
   const cmsd::U4 sw = cmsd::philox4x32_10(cmsd::U4{0u, (uint32_t)row, it, kGenSpike}, k0, k1);
   const int spike = (int)(((uint64_t)sw.x * (uint64_t)V) >> 32);
-  float* dz = draft + (size_t)row * V;
-  float* tz = target + (size_t)row * V;
+  float* dz = draft + ((size_t)b * K_max + i) * V;
+  float* tz = target + ((size_t)b * Kt + i) * V;
 
   float best = -__int_as_float(0x7F800000);
   int bidx = 0x7FFFFFFF;
@@ -53,12 +56,13 @@ __global__ void __launch_bounds__(kThreads) gen_rows_kernel(const float* __restr
         float z = table[half16(wd, j)];
         if (v == spike) z = __fadd_rn(z, h);
         const float t = __fadd_rn(z, __fmul_rn(0.8f, table[half16(wt, j)]));
-        dz[v] = z;
+        if (has_draft) dz[v] = z;
         tz[v] = t;
         if (z > best) { best = z; bidx = v; }
       }
     }
   }
+  if (!has_draft) return;     // the verifier's extra row has no drafted token
   // block argmax, lowest index among equal maxima
   for (int o = 16; o; o >>= 1) {
     const float ob = __shfl_xor_sync(0xFFFFFFFFu, best, o);
@@ -73,20 +77,20 @@ __global__ void __launch_bounds__(kThreads) gen_rows_kernel(const float* __restr
   if (threadIdx.x == 0) {
     for (int w = 1; w < kThreads / 32; ++w)
       if (sb[w] > best || (sb[w] == best && si[w] < bidx)) { best = sb[w]; bidx = si[w]; }
-    tokens[row] = bidx;
+    tokens[(size_t)b * K_max + i] = bidx;
   }
 }
 
 }  // namespace
 
 extern "C" int cmsd_gen_decode_rows(const float* table, const float* heights_it, uint32_t it, int B,
-                                    int K_max, int V, const int32_t* k_row, uint64_t seed,
+                                    int K_max, int Kt, int V, const int32_t* k_row, uint64_t seed,
                                     float* draft, float* target, int32_t* tokens, void* stream) {
-  if (B < 0 || K_max < 1 || V < 2) return -1;
+  if (B < 0 || K_max < 1 || V < 2 || (Kt != K_max && Kt != K_max + 1)) return -1;
   if (B == 0) return 0;
   if (!table || !heights_it || !draft || !target || !tokens) return -1;
-  gen_rows_kernel<<<B * K_max, kThreads, 0, (cudaStream_t)stream>>>(
-      table, heights_it, it, B, K_max, V, k_row, cmsd::seed_lo(seed), cmsd::seed_hi(seed), draft,
+  gen_rows_kernel<<<B * Kt, kThreads, 0, (cudaStream_t)stream>>>(
+      table, heights_it, it, B, K_max, Kt, V, k_row, cmsd::seed_lo(seed), cmsd::seed_hi(seed), draft,
       target, tokens);
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }

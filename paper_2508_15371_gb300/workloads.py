@@ -348,10 +348,11 @@ def ar1_heights(B, iterations, seed=4, table=None):
 def decode_row_host(table, heights, it, b, i, K_max, V, seed=4):
     """One c5 row (b, i) at iteration it: (drafter f32[V], target f32[V], drafted token).
 
-    drafter z = n1 + h[it, b] at the spike token; target = z + 0.8 * n2 (float32,
-    multiply then add); drafted token = first argmax of z.
+    Generator row id b * (K_max + 1) + i (room for the verifier's extra row at
+    i = K_max).  drafter z = n1 + h[it, b] at the spike token; target = z +
+    0.8 * n2 (float32, multiply then add); drafted token = first argmax of z.
     """
-    row = b * K_max + i
+    row = b * (K_max + 1) + i
     n1 = table[_u16_stream(seed, row, it, GEN_DNOISE, V)]
     n2 = table[_u16_stream(seed, row, it, GEN_TNOISE, V)]
     w0, _, _, _ = _philox_np(np.uint64(0), row, it, GEN_SPIKE, seed & MASK32, seed >> 32)
@@ -362,11 +363,16 @@ def decode_row_host(table, heights, it, b, i, K_max, V, seed=4):
     return z, tgt, int(np.argmax(z))
 
 
-def decode_iteration_host(table, heights, it, b, k, K_max, V, seed=4):
-    """Rows i < k of sequence b at iteration it: arrays [k, V] and tokens [k]."""
+def decode_iteration_host(table, heights, it, b, k, K_max, V, seed=4, bonus=False):
+    """Rows i < k of sequence b at iteration it: drafter [k, V], target
+    [k, V] (or [k + 1, V] with the verifier's extra row) and tokens [k]."""
+    kt = k + 1 if bonus else k
     d = np.empty((k, V), np.float32)
-    t = np.empty((k, V), np.float32)
+    t = np.empty((kt, V), np.float32)
     tok = np.empty(k, np.int64)
-    for i in range(k):
-        d[i], t[i], tok[i] = decode_row_host(table, heights, it, b, i, K_max, V, seed)
+    for i in range(kt):
+        di, ti, ki = decode_row_host(table, heights, it, b, i, K_max, V, seed)
+        t[i] = ti
+        if i < k:
+            d[i], tok[i] = di, ki
     return d, t, tok

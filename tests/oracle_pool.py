@@ -75,7 +75,7 @@ def _decode_task(task):
     heights = W.ar1_heights(B, iterations, seed, table)
 
     def gen(it, bb, k):
-        return W.decode_iteration_host(table, heights, it, bb, k, K, V, seed)
+        return W.decode_iteration_host(table, heights, it, bb, k, K, V, seed, bonus=bool(pdict.get("bonus")))
 
     return b, O.decode_sim_sequence(gen, b, iterations, K, O.Params(**pdict), seed)
 
