@@ -450,8 +450,11 @@ struct EvenSplit {
 // into warp slices.  When there are at least as many warps as rows, each row
 // is cut into wpr pieces of one warp each (no slice crosses a row end, so
 // every warp streams one segment); otherwise the stream is cut into W equal
-// runs of 16-byte vectors.  Slices start on multiples of VEC elements (the
-// last one ends at N).
+// runs of 128-byte lines.  Slices start on multiples of 128 bytes from the
+// row (or stream) start, so that a warp's 512-byte loads cover whole 32-byte
+// sectors when the rows themselves are 128-byte aligned; a 16-byte offset
+// would make every load touch one sector more (the last slice ends at N).
+constexpr int kLineVecs = 8;   // 16-byte vectors per 128-byte line
 struct StreamSplit {
   int64_t N;
   int W;          // warps with work
@@ -482,7 +485,7 @@ struct StreamSplit {
       wpr = 0;
       W = Wmax;
       qv = rv = 0;
-      const int64_t nv = N / VEC;
+      const int64_t nv = N / (VEC * kLineVecs);
       q = div_nn(nv, W);
       rem = (int)(nv - q * W);
     }
@@ -492,9 +495,9 @@ struct StreamSplit {
     if (wpr > 0) {
       const int row = w / wpr, k = w - row * wpr;
       const int off = k * qv + (k < rv ? k : rv);
-      return (int64_t)row * V + (off & ~(VEC - 1));
+      return (int64_t)row * V + (off & ~(VEC * kLineVecs - 1));
     }
-    return ((int64_t)w * q + (w < rem ? w : rem)) * VEC;
+    return ((int64_t)w * q + (w < rem ? w : rem)) * VEC * kLineVecs;
   }
   // warps holding the first and the last element of row ar
   __device__ int first_warp(int ar) const { return wpr > 0 ? ar * wpr : owner_flat((int64_t)ar * V); }
@@ -502,7 +505,7 @@ struct StreamSplit {
     return wpr > 0 ? ar * wpr + wpr - 1 : owner_flat((int64_t)ar * V + V - 1);
   }
   __device__ int owner_flat(int64_t e) const {
-    const int64_t ev = e / VEC;
+    const int64_t ev = e / (VEC * kLineVecs);
     const int64_t big = (q + 1) * rem;
     const int w = ev < big ? (int)div_nn(ev, q + 1) : rem + (int)div_nn(ev - big, q);
     return w < W ? w : W - 1;
@@ -844,11 +847,26 @@ __device__ void seg_finish(const StreamArgs& a, SegState& ss, int ar, int r, int
   constexpr bool HAS_D = MODE != kModeVerify;
   constexpr bool HAS_T = MODE != kModeConf;
   const Workspace& W = a.ws;
-  // every lane requests the 16-byte vector in which its own maximum first
-  // appeared before the warp reductions, so the load overlaps the shuffles
+  // The exact index of a lane's maximum inside its first 16-byte vector needs
+  // that vector again.  Under the sampled rule only the lanes holding the
+  // segment maximum request it (one sector each, usually one lane; this saved
+  // 19 MB of the 263 MB per launch at B=64 K=8 V=128256 and 2 us).  Under the
+  // PAPER rule every lane requests its vector before the warp reductions, so
+  // the loads overlap the shuffles: there the kernel's tail is this latency,
+  // and the early requests measured 3 us faster than the late ones.
+  const float me = HAS_D ? d_mexp(ss.d) : 0.f;
   uint4 dq = make_uint4(0, 0, 0, 0), tq = make_uint4(0, 0, 0, 0);
-  if (HAS_D && ss.d.posw > 1) dq = __ldcg(reinterpret_cast<const uint4*>(dp + ss.d.pos));
-  if (HAS_T && ss.t.posw > 1) tq = __ldcg(reinterpret_cast<const uint4*>(tp + ss.t.pos));
+  if (!SAMPLED) {
+    if (HAS_D && ss.d.posw > 1) dq = __ldcg(reinterpret_cast<const uint4*>(dp + ss.d.pos));
+    if (HAS_T && ss.t.posw > 1) tq = __ldcg(reinterpret_cast<const uint4*>(tp + ss.t.pos));
+  }
+  const float Md = HAS_D ? warp_max(me) : 0.f;
+  const float Mt = HAS_T ? warp_max(ss.t.M) : 0.f;
+  const bool dhit = HAS_D && me == Md && ss.d.posw, thit = HAS_T && ss.t.M == Mt && ss.t.posw;
+  if (SAMPLED) {
+    if (dhit && ss.d.posw > 1) dq = __ldcg(reinterpret_cast<const uint4*>(dp + ss.d.pos));
+    if (thit && ss.t.posw > 1) tq = __ldcg(reinterpret_cast<const uint4*>(tp + ss.t.pos));
+  }
   DRed dr = dred_empty();
   TRed tr = tred_empty();
   if (HAS_D) {
@@ -862,17 +880,14 @@ __device__ void seg_finish(const StreamArgs& a, SegState& ss, int ar, int r, int
     }
     float s, t2;
     d_final(d, s, t2);
-    const float me = d_mexp(d);
-    const float M = warp_max(me);
     int idx = kIntMax;
-    if (me == M && d.posw) idx = d.posw > 1 ? d.pos + first_in_vec<T>(dq, me, true) : d.pos;
+    if (dhit) idx = d.posw > 1 ? d.pos + first_in_vec<T>(dq, me, true) : d.pos;
     dr = reduce_d(DRed{me, s, t2, top2, idx});
   }
   if (HAS_T) {
     const TLane& t = ss.t;
-    const float M = warp_max(t.M);
     int idx = kIntMax;
-    if (t.M == M && t.posw) idx = t.posw > 1 ? t.pos + first_in_vec<T>(tq, t.M, false) : t.pos;
+    if (thit) idx = t.posw > 1 ? t.pos + first_in_vec<T>(tq, t.M, false) : t.pos;
     tr = reduce_t(TRed{t.M, SAMPLED ? t_final(t) : 0.f, idx, t.cnt});
   }
   // lane 0 stores the partial and counts it with a release; the warp that
