@@ -483,6 +483,14 @@ def run_ours(args):
     dev = torch.device("cuda", torch.cuda.current_device())
     peak, peak_src = peaks()
 
+    if args.only:
+        # one workload's device-resident timing, nothing else (for profiling a
+        # single configuration's launches)
+        steps = max(3, args.steps)
+        size = {"B": args.batch} if args.batch else {}
+        print(json.dumps(bench_workload(cmsd, torch, dev, args.only, args.rule, steps, peak, **size)), flush=True)
+        return 0
+
     # ---- inputs (host generation, then resident in HBM) ---------------------
     t_gen = time.perf_counter()
     sets = make_sets(rank)
@@ -678,6 +686,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-decode-sim", action="store_true", help="skip the decode-loop simulation report")
     ap.add_argument("--no-extra", action="store_true", help="headline only (no other workloads, no decode loop)")
+    ap.add_argument("--only", choices=["c1", "c2", "c3", "c4"], default=None,
+                    help="time one workload under --rule and print its object only (for profiling)")
+    ap.add_argument("--batch", type=int, default=0, help="with --only: the number of sequences B (default: full)")
     ap.add_argument("--load-window", type=float, default=0.8,
                     help="seconds of untimed steps just before the timed region (clock sampling)")
     args = ap.parse_args()
