@@ -203,9 +203,9 @@ int cmsd_confidence_verify(const void* draft_logits, const void* target_logits,
  * It allocates nothing.
  *   - Arguments and outputs: as cmsd_confidence_verify, minus ws / ws_bytes.
  *   - Limit: a problem whose cmsd_workspace_bytes(B, K, V) exceeds
- *     CMSD_STATIC_SCRATCH_BYTES (4 MiB; on a 152-SM GB300 at V = 128256 that
- *     admits about 1,000 sequences of K = 8, and B*K up to about 20,000
- *     positions at V = 32000) is rejected with CMSD_ESCRATCH, after the other
+ *     CMSD_STATIC_SCRATCH_BYTES (4 MiB; the size does not depend on V, and on
+ *     a 152-SM GB300 it admits B*K up to about 40,000 positions, e.g. about
+ *     4,900 sequences of K = 8) is rejected with CMSD_ESCRATCH, after the other
  *     argument checks and before anything is enqueued.
  *   - Each call first zero-fills, on `stream`, the part of the scratch that
  *     its layout uses, so device-side error flags (cmsd_workspace_errors) of
