@@ -432,3 +432,41 @@ def test_full_size_c3(cmsd, full_c3, rule, kw):
 @pytest.mark.parametrize("rule,kw", RULES)
 def test_full_size_c4(cmsd, full_c4, rule, kw):
     _full_size(cmsd, full_c4, "c4", rule, kw)
+
+
+def _first_sequences(W, w, n):
+    from paper_2508_15371_gb300.workloads import Workload
+    return Workload(w.name, n, w.K, w.V, w.dtype, np.ascontiguousarray(w.draft[:n]),
+                    np.ascontiguousarray(w.target[:n]), np.ascontiguousarray(w.tokens[:n]), w.seed)
+
+
+@pytest.mark.parametrize("rule,kw", RULES)
+@pytest.mark.parametrize("name,size,n", [
+    ("c3", dict(B=64), (8, 1)),               # 7 warp pieces per row, then 57 and 62
+    ("c2", dict(B=512, V=8192), (8, 1)),      # flat split over 4096 rows, then 4 pieces per row
+])
+def test_split_invariance(cmsd, W, name, size, n, rule, kw):
+    # The merge of a row's per-warp partials does not depend on how the row is
+    # cut: the same sequences inside a large batch and alone (different warp
+    # splits) give the same signals to within fp32 reordering, the same argmax
+    # and the same decisions (sequences the oracle flags as near a threshold
+    # excepted).
+    w = W.make(name, **size)
+    p = cmsd.params(w.K, rule, **kw)
+    big = gpu_fused(cmsd, torch, w, p, iteration=5)
+    for m in n:
+        ws = _first_sequences(W, w, m)
+        small = gpu_fused(cmsd, torch, ws, p, iteration=5)
+        r = oracle_fused(ws, p, iteration=5)
+        for name_ in ("H", "margin", "conf", "lse"):
+            d = np.abs(small[name_].astype(np.float64) - big[name_][:m])
+            assert np.all(np.isfinite(small[name_]) == np.isfinite(big[name_][:m]))
+            fin = np.isfinite(small[name_])
+            assert d[fin].max(initial=0.0) <= 4e-6, (name_, m, float(d[fin].max()))
+        assert np.array_equal(small["argmax"], big["argmax"][:m])
+        for b in range(m):
+            if r.k_flag[b] or r.n_flag[b] or r.tok_flag[b]:
+                continue
+            assert small["k_next"][b] == big["k_next"][b], (m, b)
+            assert small["n_accept"][b] == big["n_accept"][b], (m, b)
+            assert np.array_equal(small["out_tokens"][b], big["out_tokens"][b]), (m, b)
