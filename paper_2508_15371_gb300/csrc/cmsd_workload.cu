@@ -13,7 +13,7 @@ namespace {
 constexpr uint32_t kGenDNoise = 0xC0000002u;
 constexpr uint32_t kGenTNoise = 0xC0000003u;
 constexpr uint32_t kGenSpike = 0xC0000004u;
-constexpr int kThreads = 256;
+constexpr int kThreads = 1024;   // one row per CTA; most slots of a window are idle
 
 __device__ __forceinline__ uint32_t half16(const cmsd::U4& w, int j) {
   const uint32_t word = (j >> 1) == 0 ? w.x : (j >> 1) == 1 ? w.y : (j >> 1) == 2 ? w.z : w.w;
@@ -46,19 +46,39 @@ __global__ void __launch_bounds__(kThreads) gen_rows_kernel(const float* __restr
   float best = -__int_as_float(0x7F800000);
   int bidx = 0x7FFFFFFF;
   const int ngrp = (V + 7) / 8;
+  // rows start on 16-byte boundaries when V is a multiple of 4: each thread
+  // then writes its 8 logits as two 16-byte stores
+  const bool vec = (V & 3) == 0;
   for (int g = threadIdx.x; g < ngrp; g += kThreads) {
     const cmsd::U4 wd = cmsd::philox4x32_10(cmsd::U4{(uint32_t)g, (uint32_t)row, it, kGenDNoise}, k0, k1);
     const cmsd::U4 wt = cmsd::philox4x32_10(cmsd::U4{(uint32_t)g, (uint32_t)row, it, kGenTNoise}, k0, k1);
+    float zs[8], ts[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int v = 8 * g + j;
-      if (v < V) {
-        float z = table[half16(wd, j)];
-        if (v == spike) z = __fadd_rn(z, h);
-        const float t = __fadd_rn(z, __fmul_rn(0.8f, table[half16(wt, j)]));
-        if (has_draft) dz[v] = z;
-        tz[v] = t;
-        if (z > best) { best = z; bidx = v; }
+      float z = table[half16(wd, j)];
+      if (v == spike) z = __fadd_rn(z, h);
+      zs[j] = z;
+      ts[j] = __fadd_rn(z, __fmul_rn(0.8f, table[half16(wt, j)]));
+      if (v < V && z > best) { best = z; bidx = v; }
+    }
+    if (vec && 8 * g + 8 <= V) {
+      float4* d4 = reinterpret_cast<float4*>(dz + 8 * g);
+      float4* t4 = reinterpret_cast<float4*>(tz + 8 * g);
+      if (has_draft) {
+        d4[0] = make_float4(zs[0], zs[1], zs[2], zs[3]);
+        d4[1] = make_float4(zs[4], zs[5], zs[6], zs[7]);
+      }
+      t4[0] = make_float4(ts[0], ts[1], ts[2], ts[3]);
+      t4[1] = make_float4(ts[4], ts[5], ts[6], ts[7]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int v = 8 * g + j;
+        if (v < V) {
+          if (has_draft) dz[v] = zs[j];
+          tz[v] = ts[j];
+        }
       }
     }
   }
