@@ -562,34 +562,49 @@ def run_ours(args):
         ht = cmsd.to_device_logits(w.target, w.dtype, "cpu").pin_memory()
         hk = torch.from_numpy(w.tokens).pin_memory()
         host.append((hd, ht, hk))
-    dbuf = [(torch.empty_like(h[0], device=dev), torch.empty_like(h[1], device=dev),
-             torch.empty_like(h[2], device=dev)) for h in host[:1]]
-    ecall = cmsd.FusedCall(dbuf[0][0], dbuf[0][1], dbuf[0][2], p, seed=w0.seed, out=out, ws=ws)
+    # two device input buffers: step j+1's inputs are copied (on a copy
+    # stream) while step j computes; each step still copies all of its
+    # inputs and reads its results back inside the timed region
+    dbuf = [(torch.empty_like(host[0][0], device=dev), torch.empty_like(host[0][1], device=dev),
+             torch.empty_like(host[0][2], device=dev)) for _ in range(2)]
+    ecalls = [cmsd.FusedCall(db[0], db[1], db[2], p, seed=w0.seed, out=out, ws=ws) for db in dbuf]
     res_host = [torch.empty(B, dtype=torch.int32).pin_memory(), torch.empty((B, K), dtype=torch.int32).pin_memory(),
                 torch.empty(B, dtype=torch.int32).pin_memory()]
     h2d = sum(x.numel() * x.element_size() for x in host[0])
     d2h = sum(x.numel() * x.element_size() for x in res_host)
+    main = torch.cuda.current_stream()
+    cs = torch.cuda.Stream()
+    copied = [torch.cuda.Event() for _ in range(2)]
+    computed = [torch.cuda.Event() for _ in range(2)]
 
-    def e2e_step(j):
-        hd, ht, hk = host[j % len(host)]
-        dbuf[0][0].copy_(hd, non_blocking=True)
-        dbuf[0][1].copy_(ht, non_blocking=True)
-        dbuf[0][2].copy_(hk, non_blocking=True)
-        o = ecall(iteration=j)
-        res_host[0].copy_(o["n_accept"], non_blocking=True)
-        res_host[1].copy_(o["out_tokens"], non_blocking=True)
-        res_host[2].copy_(o["k_next"], non_blocking=True)
+    def e2e_steps_run(n, start_event=None):
+        if start_event is not None:
+            cs.wait_event(start_event)
+        for j in range(n):
+            hd, ht, hk = host[j % len(host)]
+            db = dbuf[j % 2]
+            with torch.cuda.stream(cs):
+                if j >= 2:
+                    cs.wait_event(computed[j % 2])     # the buffer's previous step is done
+                db[0].copy_(hd, non_blocking=True)
+                db[1].copy_(ht, non_blocking=True)
+                db[2].copy_(hk, non_blocking=True)
+                copied[j % 2].record(cs)
+            main.wait_event(copied[j % 2])
+            o = ecalls[j % 2](iteration=j)
+            res_host[0].copy_(o["n_accept"], non_blocking=True)
+            res_host[1].copy_(o["out_tokens"], non_blocking=True)
+            res_host[2].copy_(o["k_next"], non_blocking=True)
+            computed[j % 2].record(main)
 
-    for j in range(3):
-        e2e_step(j)
+    e2e_steps_run(3)
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record()
-    for j in range(e2e_steps):
-        e2e_step(j)
+    e2e_steps_run(e2e_steps, start_event=e0)
     e1.record()
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), dist, dev)
@@ -661,6 +676,8 @@ def run_ours(args):
         "resample_ms": statistics.median(r_ms) if sampled else 0.0,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "overlap": "step j+1's host-to-device copies run on a copy stream during step j's pass "
+                           "(two device input buffers)",
                 "steps": e2e_steps},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk,
