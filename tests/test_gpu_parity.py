@@ -470,3 +470,39 @@ def test_split_invariance(cmsd, W, name, size, n, rule, kw):
             assert small["k_next"][b] == big["k_next"][b], (m, b)
             assert small["n_accept"][b] == big["n_accept"][b], (m, b)
             assert np.array_equal(small["out_tokens"][b], big["out_tokens"][b]), (m, b)
+
+
+@pytest.mark.parametrize("rule,kw", RULES)
+def test_parity_max_window(cmsd, W, rule, kw):
+    # K = 1024, the largest window: the epilogue takes the per-row path
+    w = W.make("c2", B=2, K=1024, V=96, dtype="f32")
+    p = cmsd.params(w.K, rule, **kw)
+    compare(w, gpu_fused(cmsd, torch, w, p, iteration=2), oracle_fused(w, p, iteration=2))
+
+
+@pytest.mark.parametrize("rule,kw", RULES)
+def test_parity_ragged_max_batch(cmsd, W, rule, kw):
+    # B = 12000 sequences with a k_row (the largest ragged batch), windows of
+    # 0..4 positions; every 97th sequence against the oracle, invariants on all
+    import oracle_pool
+    w = W.make("c2", B=12000, K=4, V=136, dtype="bf16")
+    k_row = np.random.default_rng(12).integers(0, 5, w.B).astype(np.int32)
+    p = cmsd.params(w.K, rule, **kw)
+    g = gpu_fused(cmsd, torch, w, p, iteration=4, k_row=k_row)
+    seqs = list(range(0, w.B, 97))
+    r = oracle_pool.fused(w, p.as_dict(), w.seed, iteration=4, k_row=k_row, seqs=seqs)
+    compare(w, g, r, k_row=k_row, seqs=seqs)
+    n, k = g["n_accept"], g["k_next"]
+    assert np.all((n >= 0) & (n <= k_row))
+    assert np.all((k >= p.k_min) & (k <= p.k_max))
+    for b in np.where(k_row == 0)[0]:
+        assert n[b] == 0 and np.all(g["out_tokens"][b] == -1)
+
+
+@pytest.mark.parametrize("rule,kw", RULES)
+def test_parity_large_vocab(cmsd, W, rule, kw):
+    # V = 1,000,003 (odd: unaligned rows, scalar heads and tails), about 127
+    # warp pieces per row
+    w = W.make("c2", B=1, K=3, V=1000003, dtype="f32")
+    p = cmsd.params(w.K, rule, **kw)
+    compare(w, gpu_fused(cmsd, torch, w, p, iteration=9), oracle_fused(w, p, iteration=9))
