@@ -9,7 +9,7 @@
  * paper's drafter and verifier models (Sec. IV.A), which are not available.
  *
  * Row (b, i) at iteration `it` (row id r = b * (K_max + 1) + i):
- *   n1[v], n2[v] = table[u16] with u16 the 16-bit half (v & 1) of Philox4x32-10
+ *   n1[v], n2[v] = table[u16 >> 3] with u16 the 16-bit half (v & 1) of Philox4x32-10
  *                  word (v >> 1) & 3 of counter (v >> 3, r, it, 0xC0000002 / 0xC0000003),
  *                  key (seed lo, seed hi)
  *   spike token  = (word 0 of counter (0, r, it, 0xC0000004)) * V >> 32
@@ -28,7 +28,7 @@
 extern "C" {
 #endif
 
-/* table: float[65536] device (normal quantiles); heights_it: float[B] device
+/* table: float[8192] device (normal quantiles at (j + 1/2) / 8192); heights_it: float[B] device
  * (spike heights of this iteration); k_row: int32[B] device (NULL = K_max);
  * Kt: verifier rows per sequence, K_max or K_max + 1;
  * draft: float [B][K_max][V] device; target: float [B][Kt][V] device;

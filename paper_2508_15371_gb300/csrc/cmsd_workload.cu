@@ -14,6 +14,7 @@ constexpr uint32_t kGenDNoise = 0xC0000002u;
 constexpr uint32_t kGenTNoise = 0xC0000003u;
 constexpr uint32_t kGenSpike = 0xC0000004u;
 constexpr int kThreads = 1024;   // one row per CTA; most slots of a window are idle
+constexpr int kTableBits = 13;   // the normal table: 2^13 float32, staged in shared memory
 
 __device__ __forceinline__ uint32_t half16(const cmsd::U4& w, int j) {
   const uint32_t word = (j >> 1) == 0 ? w.x : (j >> 1) == 1 ? w.y : (j >> 1) == 2 ? w.z : w.w;
@@ -36,6 +37,9 @@ __global__ void __launch_bounds__(kThreads) gen_rows_kernel(const float* __restr
   }
   const bool has_draft = i < k;
   if (!has_draft && i >= k + (Kt - K_max)) return;
+  __shared__ float s_table[1 << kTableBits];
+  for (int j = threadIdx.x; j < (1 << kTableBits); j += kThreads) s_table[j] = table[j];
+  __syncthreads();
   const int row = b * (K_max + 1) + i;          // generator row id
   const float h = heights_it[b];
   const cmsd::U4 sw = cmsd::philox4x32_10(cmsd::U4{0u, (uint32_t)row, it, kGenSpike}, k0, k1);
@@ -56,10 +60,10 @@ __global__ void __launch_bounds__(kThreads) gen_rows_kernel(const float* __restr
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int v = 8 * g + j;
-      float z = table[half16(wd, j)];
+      float z = s_table[half16(wd, j) >> (16 - kTableBits)];
       if (v == spike) z = __fadd_rn(z, h);
       zs[j] = z;
-      ts[j] = __fadd_rn(z, __fmul_rn(0.8f, table[half16(wt, j)]));
+      ts[j] = __fadd_rn(z, __fmul_rn(0.8f, s_table[half16(wt, j) >> (16 - kTableBits)]));
       if (v < V && z > best) { best = z; bidx = v; }
     }
     if (vec && 8 * g + 8 <= V) {

@@ -300,11 +300,15 @@ def _philox_np(c0, c1, c2, c3, k0, k1):
     return c0, c1, c2, c3
 
 
-def normal_table(bits=16):
+NORMAL_BITS = 13          # the table's size: 2**13 float32 (32 KB, held in shared memory on the device)
+
+
+def normal_table(bits=NORMAL_BITS):
     """Quantiles of N(0,1) at the midpoints (k + 1/2) / 2**bits, as float32.
 
-    A 16-bit uniform indexes it, giving a discretised normal that host and
-    device reproduce exactly (a table lookup, no transcendental calls).
+    The top `bits` bits of a 16-bit uniform index it, giving a discretised
+    normal that host and device reproduce exactly (a table lookup, no
+    transcendental calls).
     """
     from scipy.special import ndtri
     n = 1 << bits
@@ -338,7 +342,7 @@ def ar1_heights(B, iterations, seed=4, table=None):
     b = np.arange(B, dtype=np.uint64)
     for it in range(iterations):
         w0, _, _, _ = _philox_np(np.uint64(0), b, it, GEN_AR, seed & MASK32, seed >> 32)
-        eps = table[(w0 & np.uint64(0xFFFF)).astype(np.int64)]
+        eps = table[((w0 & np.uint64(0xFFFF)) >> np.uint64(16 - NORMAL_BITS)).astype(np.int64)]
         h = (rho * h + c) + sg * eps
         h = np.minimum(np.float32(C5_HMAX), np.maximum(np.float32(0.0), h)).astype(np.float32)
         out[it] = h
@@ -353,8 +357,8 @@ def decode_row_host(table, heights, it, b, i, K_max, V, seed=4):
     0.8 * n2 (float32, multiply then add); drafted token = first argmax of z.
     """
     row = b * (K_max + 1) + i
-    n1 = table[_u16_stream(seed, row, it, GEN_DNOISE, V)]
-    n2 = table[_u16_stream(seed, row, it, GEN_TNOISE, V)]
+    n1 = table[_u16_stream(seed, row, it, GEN_DNOISE, V) >> (16 - NORMAL_BITS)]
+    n2 = table[_u16_stream(seed, row, it, GEN_TNOISE, V) >> (16 - NORMAL_BITS)]
     w0, _, _, _ = _philox_np(np.uint64(0), row, it, GEN_SPIKE, seed & MASK32, seed >> 32)
     tok = int((int(w0) * V) >> 32)
     z = n1.copy()

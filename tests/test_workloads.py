@@ -44,7 +44,7 @@ def test_c3_profile_readings():
 
 def test_c5_generator_tables():
     t = W.normal_table()
-    assert t.shape == (65536,) and t.dtype == np.float32
+    assert t.shape == (1 << W.NORMAL_BITS,) == (8192,) and t.dtype == np.float32
     assert np.all(np.diff(t) > 0) and abs(float(t.mean())) < 1e-6
     assert float(t.std()) == pytest.approx(1.0, abs=2e-3)
     h = W.ar1_heights(32, 200, seed=4, table=t)
