@@ -1221,6 +1221,31 @@ __device__ __forceinline__ int race_group_entries(uint4 qt, uint4 qd, int gm, in
   return km != pos_inf() ? vm : -1;
 }
 
+// Units (queued row rr, group g) -> u = rr * ng + g, split over Weff warps.
+// When every queued row can have a warp, each row gets wpr warps of its own:
+// no warp's units then cross a row end, which would make it stage, race and
+// merge two rows one after the other.  Otherwise the units are split evenly
+// in order.
+struct ResSplit {
+  int R, ng, wpr;
+  EvenSplit by_row;   // a row's ng groups over its wpr warps
+  EvenSplit flat;     // all units over Weff warps
+  __device__ ResSplit(int R_, int ng_, int Weff)
+      : R(R_), ng(ng_), wpr(R_ <= Weff ? Weff / R_ : 0), by_row(ng_, wpr > 0 ? wpr : 1),
+        flat((int64_t)R_ * ng_, Weff) {}
+  __device__ int64_t start(int w) const {
+    if (wpr == 0) return flat.start(w);
+    if (w >= R * wpr) return (int64_t)R * ng;
+    const int rr = w / wpr;
+    return (int64_t)rr * ng + by_row.start(w - rr * wpr);
+  }
+  __device__ int owner(int64_t u) const {
+    if (wpr == 0) return flat.owner(u);
+    const int rr = (int)div_nn(u, ng);
+    return rr * wpr + by_row.owner(u - (int64_t)rr * ng);
+  }
+};
+
 #ifndef CMSD_RES_MIN_BLOCKS
 #define CMSD_RES_MIN_BLOCKS 3
 #endif
@@ -1235,26 +1260,58 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 // The groups [gc, ge) of one row (target, and drafter when `two`) into this
-// warp's stage: the vectors wholly inside the row go by cp.async, all in
-// flight together; returns how many (the rest is read element by element).
+// warp's stage, as a series of cp.async groups of kResSubIters race
+// iterations each, all in flight together: the race over the first part of
+// the stage starts while the rest is still arriving.  Only vectors wholly
+// inside the row go by cp.async (the rest is read element by element);
+// returns how many, and the number of cp.async groups committed in nsub.
+#ifndef CMSD_RES_SUB_ITERS
+#define CMSD_RES_SUB_ITERS 2
+#endif
+constexpr int kResSubIters = CMSD_RES_SUB_ITERS;
 template <typename T>
 __device__ __forceinline__ int stage_groups(const T* tp, const T* dp, bool two, int gc, int ge, int V, bool vec_ok,
-                                            uint32_t st_t, uint32_t st_d, int lane) {
+                                            uint32_t st_t, uint32_t st_d, int lane, int& nsub) {
   constexpr int VEC = Elem<T>::kVec;
   constexpr int LPG = kGroup / VEC;
+  constexpr int GPI = 32 / LPG;
+  constexpr int SG = kResSubIters * GPI;    // groups per cp.async group
   const int v_base = gc * kGroup;
   const int nfull = vec_ok ? min((ge - gc) * LPG, (V - v_base) / VEC) : 0;
-  for (int j = lane; j < nfull; j += 32) {
-    cp_async16(st_t + 16u * (uint32_t)j, tp + v_base + j * VEC);
-    if (two) cp_async16(st_d + 16u * (uint32_t)j, dp + v_base + j * VEC);
+  const int ns = (ge - gc + SG - 1) / SG;
+  for (int k = 0; k < ns; ++k) {
+#pragma unroll
+    for (int m = 0; m < kResSubIters; ++m) {
+      const int j = (k * kResSubIters + m) * 32 + lane;    // 32 vectors per race iteration
+      if (j < nfull) {
+        cp_async16(st_t + 16u * (uint32_t)j, tp + v_base + j * VEC);
+        if (two) cp_async16(st_d + 16u * (uint32_t)j, dp + v_base + j * VEC);
+      }
+    }
+    cp_async_commit();
   }
-  cp_async_commit();
-  cp_async_wait_all();
-  __syncwarp();
+  nsub = ns;
   return nfull;
+}
+
+// Wait until at most `pending` of this thread's latest cp.async groups are in
+// flight, then make the whole warp's completed copies visible to the warp.
+__device__ __forceinline__ void stage_wait(int pending) {
+  switch (pending) {
+    case 0: asm volatile("cp.async.wait_group 0;" ::: "memory"); break;
+    case 1: asm volatile("cp.async.wait_group 1;" ::: "memory"); break;
+    case 2: asm volatile("cp.async.wait_group 2;" ::: "memory"); break;
+    case 3: asm volatile("cp.async.wait_group 3;" ::: "memory"); break;
+    case 4: asm volatile("cp.async.wait_group 4;" ::: "memory"); break;
+    case 5: asm volatile("cp.async.wait_group 5;" ::: "memory"); break;
+    case 6: asm volatile("cp.async.wait_group 6;" ::: "memory"); break;
+    default: asm volatile("cp.async.wait_group 7;" ::: "memory"); break;
+  }
+  __syncwarp();
 }
 
 // Vector `sub` of group g (staged chunk starting at group gc), or -inf
@@ -1276,6 +1333,11 @@ __global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_ker
   constexpr int LPG = kGroup / VEC;    // lanes per group
   constexpr int GPI = 32 / LPG;        // groups per warp iteration
   constexpr int CG = kResStageBytes / (2 * kGroup * (int)sizeof(T));   // groups per stage
+  static_assert(CG / (kResSubIters * GPI) <= 8, "stage_wait covers at most 8 cp.async groups");
+  constexpr int SG = kResSubIters * GPI;            // groups per sub-stage of the sampled race's ring
+  constexpr int SV = kResSubIters * 32;             // 16-byte vectors per sub-stage and tensor
+  constexpr int NSLOT = CG / SG;                    // sub-stages in the ring
+  static_assert(NSLOT >= 2 && NSLOT * SV * 16 == kResStageBytes / 2, "ring layout");
   extern __shared__ __align__(16) unsigned char res_smem[];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
@@ -1294,7 +1356,7 @@ __global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_ker
     const int Weff = (int)(want < 1 ? 1 : (want > a.nwarps ? a.nwarps : want));
     const int w = blockIdx.x * kResWarps + warp;
     if (w < Weff) {
-      const EvenSplit sp(NU, Weff);
+      const ResSplit sp(R, ng, Weff);
       int64_t u0 = sp.start(w);
       const int64_t u1 = sp.start(w + 1);
       const uint32_t k0 = seed_lo(a.seed), k1 = seed_hi(a.seed);
@@ -1329,8 +1391,11 @@ __global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_ker
           int bi = kIntMax;
           for (int gc = g0; gc < g1; gc += CG) {
             const int ge = min(g1, gc + CG);
-            const int nfull = stage_groups<T>(tp, dp, false, gc, ge, a.V, vec_ok, st_t, st_d, lane);
+            int nsub = 0;
+            const int nfull = stage_groups<T>(tp, dp, false, gc, ge, a.V, vec_ok, st_t, st_d, lane, nsub);
             for (int gi = gc; gi < ge; gi += GPI) {
+              const int itr = (gi - gc) / GPI;
+              if (itr % kResSubIters == 0) stage_wait(nsub - 1 - itr / kResSubIters);
               const int g = gi + lane / LPG;
               const uint4 qt = staged_vec<T>(stage, tp, g, gc, ge, sub, nfull, a.V);
               const int v = g * kGroup + sub * VEC;
@@ -1369,15 +1434,52 @@ __global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_ker
           uint4 bqt = neg_inf_vec<T>(), bqd = make_uint4(0, 0, 0, 0);
           int gb = -kGroupBatch;               // first group of the drawn batch
           U4 gw = U4{0u, 0u, 0u, 0u};
-          for (int gc = g0; gc < g1; gc += CG) {
-            const int ge = min(g1, gc + CG);
-            const int nfull = stage_groups<T>(tp, dp, resid_kind, gc, ge, a.V, vec_ok, st_t, st_d, lane);
-            if (resid_kind && gc == g0) st = RowStat{ts.x, 1.0f / ts.y, ds.x, -1.0f / ds.y};
-            for (int gi = gc; gi < ge; gi += GPI) {
+          // The groups [g0, g1) stream through the warp's stage as a ring of
+          // NSLOT sub-stages of SG groups: sub-stage s + NSLOT - 1 is copied
+          // while sub-stage s is raced.  Vector jr of the range (jr = 32 *
+          // race iteration + lane) is copied and read by lane jr % 32 alone,
+          // so each lane waits only for its own copies.
+          const int S = (g1 - g0 + SG - 1) / SG;
+          const int vb = g0 * kGroup;
+          const int jfull = vec_ok ? min((g1 - g0) * LPG, (a.V - vb) / VEC) : 0;
+          auto issue = [&](int sidx) {
+            if (sidx < S) {
+              const uint32_t sb = 16u * (uint32_t)((sidx % NSLOT) * SV + lane);
+#pragma unroll
+              for (int m = 0; m < kResSubIters; ++m) {
+                const int jr = (sidx * kResSubIters + m) * 32 + lane;
+                if (jr < jfull) {
+                  cp_async16(st_t + sb + 512u * (uint32_t)m, tp + vb + jr * VEC);
+                  if (resid_kind) cp_async16(st_d + sb + 512u * (uint32_t)m, dp + vb + jr * VEC);
+                }
+              }
+            }
+            cp_async_commit();              // one group per sub-stage, empty past the range
+          };
+#pragma unroll
+          for (int sidx = 0; sidx < NSLOT - 1; ++sidx) issue(sidx);
+          if (resid_kind) st = RowStat{ts.x, 1.0f / ts.y, ds.x, -1.0f / ds.y};
+          for (int sidx = 0; sidx < S; ++sidx) {
+            issue(sidx + NSLOT - 1);        // into the slot raced one sub-stage ago
+            cp_async_wait<NSLOT - 1>();     // this lane's copies of sub-stage sidx are in
+            const unsigned char* slot = stage + 16 * ((sidx % NSLOT) * SV + lane);
+#pragma unroll
+            for (int m = 0; m < kResSubIters; ++m) {
+              const int gi = g0 + (sidx * kResSubIters + m) * GPI;
+              if (gi >= g1) break;
               const int g = gi + lane / LPG;
-              const uint4 qt = staged_vec<T>(stage, tp, g, gc, ge, sub, nfull, a.V);
-              const uint4 qd = resid_kind ? staged_vec<T>(stage + kResStageBytes / 2, dp, g, gc, ge, sub, nfull, a.V)
-                                          : make_uint4(0, 0, 0, 0);
+              const int jr = (sidx * kResSubIters + m) * 32 + lane;
+              uint4 qt = neg_inf_vec<T>(), qd = make_uint4(0, 0, 0, 0);
+              if (resid_kind) qd = neg_inf_vec<T>();
+              if (g < g1) {
+                if (jr < jfull) {
+                  qt = *reinterpret_cast<const uint4*>(slot + 512 * m);
+                  if (resid_kind) qd = *reinterpret_cast<const uint4*>(slot + 512 * m + kResStageBytes / 2);
+                } else {
+                  qt = load_logits<T>(tp, vb + jr * VEC, a.V, false);
+                  if (resid_kind) qd = load_logits<T>(dp, vb + jr * VEC, a.V, false);
+                }
+              }
               if (gi + GPI > gb + kGroupBatch) {   // warp-uniform: draw the next 128 group uniforms
                 gb = gi & ~3;
                 gw = philox4x32_10(U4{(uint32_t)(gb >> 2) + (uint32_t)lane, (uint32_t)b, (uint32_t)pos, cw_grp},
@@ -1395,7 +1497,7 @@ __global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_ker
               // warp's best so far and cannot win (the factor covers the
               // rounding of E and of the product)
               bool improved = false;
-              if (g < ge && acc > 0.f && word_to_unit(word) * kRaceFilter < thr * acc) {
+              if (g < g1 && acc > 0.f && word_to_unit(word) * kRaceFilter < thr * acc) {
                 const float key = expo(word) / acc;
                 if (key < best) {          // groups are visited in increasing order
                   best = key;
@@ -1407,7 +1509,6 @@ __global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_ker
               }
               if (__any_sync(kFull, improved)) thr = warp_min(best);
             }
-            __syncwarp();                  // the stage is rewritten by the next chunk
           }
           const float kmin = warp_min(best);
           const int gmin = warp_min_i(best == kmin ? bestg : kIntMax);
