@@ -28,3 +28,4 @@ from .cmsd_oracle import (  # noqa: F401
     verify_sequence,
 )
 from . import philox  # noqa: F401
+from .lmhead import lm_head_confidence, lm_head_logits, signal_error_bound  # noqa: F401

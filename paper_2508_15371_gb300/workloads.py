@@ -253,6 +253,63 @@ def make_c4(B=256, K=16, V=152064, seed=3, dtype="bf16", threads=None):
 RECIPES = {"c1": make_c1, "c2": make_c2, "c3": make_c3, "c4": make_c4}
 
 
+# ---------------------------------------------------------------------------
+# drafter LM head: hidden states and weights (the fused LM-head entry point)
+# ---------------------------------------------------------------------------
+
+@dataclass
+class LMHeadWorkload:
+    name: str
+    R: int
+    d: int
+    V: int
+    seed: int
+    hidden: np.ndarray      # uint16 bf16 bits [R, d]
+    weight: np.ndarray      # uint16 bf16 bits [V, d]
+    spike_token: np.ndarray  # int64 [R]: the vocabulary row a hidden state points at (-1: none)
+    note: str
+
+
+def make_lmhead(R=64, d=2048, V=128256, seed=5, exact=False, spiked=0.7):
+    """Hidden states [R, d] and an LM-head weight [V, d], bf16, seeded.
+
+    Default recipe (a 1B-class drafter's head at a Llama-3-sized vocabulary):
+    W[v, j] ~ N(0, 1) / sqrt(d); each hidden state is N(0, 0.7^2) noise, and
+    with probability `spiked` also points at a uniform vocabulary row v* with
+    a height a ~ U[0, 12] (h += a W[v*] / |W[v*]|^2), so the logit at v* is
+    raised by about a: a spread from flat to peaked rows, like c1.
+
+    exact=True: every entry is a multiple of 1/16 (W in [-1/8, 1/8], h in
+    [-1/4, 1/4], a spiked row adds W[v*]), so each product is a multiple of
+    2^-8 and every partial sum of a dot product is exact in float32 for
+    d <= 2^14: float32 logits then equal the float64 ones in any order.
+    """
+    rng = np.random.default_rng(np.random.SeedSequence([seed, R, d, V, int(exact)]))
+    if exact:
+        w32 = rng.integers(-2, 3, size=(V, d)).astype(np.float32) / 16.0
+        h32 = rng.integers(-2, 3, size=(R, d)).astype(np.float32) / 16.0
+    else:
+        w32 = (rng.standard_normal((V, d), dtype=np.float32) / np.float32(np.sqrt(d))).astype(np.float32)
+        h32 = (0.7 * rng.standard_normal((R, d), dtype=np.float32)).astype(np.float32)
+    wb = f32_to_bf16_bits(w32)
+    wq = bf16_bits_to_f32(wb)
+    spike = np.full(R, -1, dtype=np.int64)
+    for r in range(R):
+        if rng.random() < spiked:
+            v = int(rng.integers(0, V))
+            spike[r] = v
+            if exact:
+                h32[r] += wq[v]
+            else:
+                a = rng.uniform(0.0, 12.0)
+                h32[r] += np.float32(a) * wq[v] / np.float32(np.dot(wq[v], wq[v]))
+    hb = f32_to_bf16_bits(h32)
+    note = ("entries are multiples of 1/16 (float32 dot products exact)" if exact else
+            "W ~ N(0,1)/sqrt(d); h ~ N(0,0.7^2) plus a spike of height U[0,12] towards a uniform token "
+            "on %.0f%% of rows" % (100 * spiked))
+    return LMHeadWorkload("lmhead", R, d, V, seed, hb, wb, spike, note)
+
+
 def make(name, **kw):
     """Full-size recipe `name`, with any size/seed overridden by keyword."""
     base = dict(FULL_SIZES[name])
