@@ -150,6 +150,35 @@ int cmsd_confidence(const void* draft_logits, int B, int K, int V, int dtype,
                     int32_t* k_next, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * The drafter's LM head fused with the confidence signals (Sec. I: the
+ * estimator is a light layer over the drafter's output logits; Sec.
+ * III.B(1): its signals).  For each of R hidden states h (one per drafted
+ * row): z = h W^T over the whole vocabulary, then the per-row outputs of
+ * cmsd_confidence (H, margin, argmax = the greedy drafted token, conf, lse)
+ * from z, without writing z to memory.
+ *   hidden: bf16 [R][d] device, row-major; weight: bf16 [V][d] device,
+ *     row-major (the [out][in] layout of a linear layer); both 16-byte
+ *     aligned; d a multiple of 64, 64 <= d <= 2^20; 2 <= V; R*V < 2^46;
+ *     R == 0 is a valid empty call.  Entries must be finite.
+ *   z is accumulated in fp32 from exact bf16 products (tensor cores), in an
+ *   order that differs from a sequential sum: each logit differs from the
+ *   exact dot product by rounding only.
+ *   H, margin, argmax, conf, lse: [R] device outputs, each may be NULL.
+ *   logits: NULL, or fp32 [R][V] device: z is also written there (for
+ *     checking; it costs R*V*4 bytes of writes).
+ *   ws: a workspace of at least cmsd_lmhead_workspace_bytes(R, d, V) bytes on
+ *     the current device (no initialisation needed; calls that share one
+ *     must be ordered on one stream).
+ * Two kernels on `stream`: the GEMM with the per-row statistics in its
+ * epilogue, then a per-row merge of the statistics of the vocabulary runs.
+ */
+size_t cmsd_lmhead_workspace_bytes(int R, int d, int V);
+int cmsd_lmhead_confidence(const void* hidden, const void* weight, int R, int d, int V,
+                           const cmsd_params* p, float* H, float* margin, int32_t* argmax,
+                           float* conf, float* lse, float* logits, void* ws, size_t ws_bytes,
+                           void* stream);
+
+/*
  * Verification (Sec. III.B(c)) given the confidence of each present position.
  * draft_tokens: int32 [B][K] device, the drafted token of each position.
  * conf: float [B][K] device, C_t (e.g. from cmsd_confidence).

@@ -21,7 +21,7 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
 
 LIBS = {
-    "libcmsd.so": ["cmsd_stream_bf16.cu", "cmsd_stream_f32.cu", "cmsd_api.cu", "cmsd_static.cu"],
+    "libcmsd.so": ["cmsd_stream_bf16.cu", "cmsd_stream_f32.cu", "cmsd_api.cu", "cmsd_static.cu", "cmsd_lmhead.cu"],
     "libcmsd_workload.so": ["cmsd_workload.cu"],
 }
 

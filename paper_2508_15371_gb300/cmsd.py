@@ -70,6 +70,9 @@ _SIGS = {
     "cmsd_confidence_verify_static": (_c_int, [_vp, _vp, _vp, _vp, _c_int, _c_int, _c_int, _c_int, _vp,
                                                _c_u64, _c_u32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                                _vp, _vp]),
+    "cmsd_lmhead_workspace_bytes": (_c_sz, [_c_int, _c_int, _c_int]),
+    "cmsd_lmhead_confidence": (_c_int, [_vp, _vp, _c_int, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp, _vp,
+                                        _vp, _vp, _c_sz, _vp]),
     "cmsd_philox_u32": (_c_u32, [_c_u64, _c_u32, _c_u32, _c_u32, _c_u32, _c_int]),
     "cmsd_philox_fill": (_c_int, [_c_u64, _c_u32, _c_u32, _c_u32, _c_u32, _vp, _c_sz, _vp]),
     "cmsd_profile_start": (_c_int, [_c_int]),
@@ -223,6 +226,43 @@ def confidence(draft, k_row=None, p=None, out=None, ws=None):
                                _ptr(o["H"]), _ptr(o["margin"]), _ptr(o["argmax"]), _ptr(o["conf"]),
                                _ptr(o["lse"]), _ptr(o["k_next"]), _ptr(ws), ws.numel(), _stream())
     _check(rc, "cmsd_confidence")
+    return o
+
+
+def lmhead_workspace(R, d, V):
+    """A workspace for cmsd_lmhead_confidence(R, d, V) on the current device."""
+    torch = _torch()
+    n = int(lib().cmsd_lmhead_workspace_bytes(R, d, V))
+    if n == 0:
+        raise CmsdError("cmsd_lmhead_workspace_bytes failed")
+    return torch.empty(n, dtype=torch.uint8, device="cuda")
+
+
+def lmhead_confidence(hidden, weight, p=None, logits=False, out=None, ws=None):
+    """The drafter's LM head fused with the confidence signals.
+
+    hidden: bf16 [R, d] (torch.bfloat16 or int16/uint16 bits), weight: bf16
+    [V, d].  Returns dict H, margin, argmax, conf, lse ([R]) and, with
+    logits=True, the fp32 logits [R, V]."""
+    torch = _torch()
+    _need_cuda(hidden, weight)
+    if hidden.element_size() != 2 or weight.element_size() != 2:
+        raise CmsdError("hidden and weight must hold 16-bit (bf16) values")
+    R, d = hidden.shape
+    V, d2 = weight.shape
+    if d2 != d:
+        raise CmsdError("hidden [R, d] and weight [V, d] must share d")
+    p = p if p is not None else params(1)
+    dev = hidden.device
+    o = {n: _out(out, n, (R,), torch.float32, dev) for n in ("H", "margin", "conf", "lse")}
+    o["argmax"] = _out(out, "argmax", (R,), torch.int32, dev)
+    if logits:
+        o["logits"] = _out(out, "logits", (R, V), torch.float32, dev)
+    ws = ws if ws is not None else lmhead_workspace(R, d, V)
+    rc = lib().cmsd_lmhead_confidence(_ptr(hidden), _ptr(weight), R, d, V, ctypes.byref(p), _ptr(o["H"]),
+                                      _ptr(o["margin"]), _ptr(o["argmax"]), _ptr(o["conf"]), _ptr(o["lse"]),
+                                      _ptr(o.get("logits")), _ptr(ws), ws.numel(), _stream())
+    _check(rc, "cmsd_lmhead_confidence")
     return o
 
 

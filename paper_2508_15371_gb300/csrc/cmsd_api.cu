@@ -306,6 +306,32 @@ int validate_fused(const void* draft_logits, const void* target_logits, const in
 
 // ============================================================ C ABI
 
+// ---------------------------------------------------------------- LM head
+
+namespace {
+struct LmLayout {
+  size_t row_conf, part, total;
+  int nct;
+};
+int lm_layout(int R, int V, LmLayout* L) {
+  int sms = 0;
+  int rc = device_sms(&sms);
+  if (rc) return rc;
+  L->nct = lmhead_ctas_per_block(sms, R, V);
+  const size_t nrb = (size_t)(R + kLhRows - 1) / kLhRows;
+  size_t o = up(sizeof(unsigned));
+  L->row_conf = o; o += up((size_t)R * sizeof(unsigned long long));
+  L->part = o; o += up(nrb * (size_t)L->nct * kLhRows * sizeof(Partial));
+  L->total = o;
+  return CMSD_OK;
+}
+int check_lmhead(int R, int d, int V) {
+  if (R < 0 || d < 64 || d % 64 != 0 || d > (1 << 20) || V < 2) return CMSD_EINVAL;
+  if ((double)R * (double)V >= 70368744177664.0) return CMSD_EINVAL;   // 2^46 logits
+  return CMSD_OK;
+}
+}  // namespace
+
 extern "C" {
 
 void cmsd_params_default(cmsd_params* p, int K, int rule) {
@@ -338,6 +364,48 @@ int cmsd_params_preset(cmsd_params* p, int K, int rule, int preset) {
     default: return CMSD_EINVAL;
   }
   return CMSD_OK;
+}
+
+
+size_t cmsd_lmhead_workspace_bytes(int R, int d, int V) {
+  if (check_lmhead(R, d, V)) return 0;
+  LmLayout L;
+  if (lm_layout(R, V, &L)) return 0;
+  return L.total;
+}
+
+int cmsd_lmhead_confidence(const void* hidden, const void* weight, int R, int d, int V,
+                           const cmsd_params* p, float* H, float* margin, int32_t* argmax, float* conf,
+                           float* lse, float* logits, void* ws, size_t ws_bytes, void* stream) {
+  int rc = check_lmhead(R, d, V);
+  if (rc) return rc;
+  rc = check_params(p, false);
+  if (rc) return rc;
+  if (R == 0) return CMSD_OK;
+  if (!hidden || !weight) return CMSD_EINVAL;
+  if (!aligned16(hidden) || !aligned16(weight)) return CMSD_EALIGN;
+  LmLayout L;
+  rc = lm_layout(R, V, &L);
+  if (rc) return rc;
+  if (!ws || ws_bytes < L.total) return CMSD_ENOWS;
+  StreamArgs a = blank_args();
+  fill_sizes(a, R, 1, V);
+  fill_params(a, p);
+  a.Kt = a.Ko = 1;
+  a.H = H; a.margin = margin; a.argmax = argmax; a.conf = conf; a.lse = lse;
+  char* w = (char*)ws;
+  a.ws.err = (unsigned*)w;
+  a.ws.row_conf = (unsigned long long*)(w + L.row_conf);
+  LmHeadArgs h;
+  h.hidden = (const uint16_t*)hidden;
+  h.weight = (const uint16_t*)weight;
+  h.R = R; h.d = d; h.V = V;
+  h.nct = L.nct;
+  h.logits = logits;
+  h.part = (Partial*)(w + L.part);
+  h.err = a.ws.err;
+  cudaError_t e = launch_lmhead(h, a, (cudaStream_t)stream);
+  return e == cudaSuccess ? CMSD_OK : cuda_fail(e);
 }
 
 size_t cmsd_workspace_bytes(int B, int K, int V) {

@@ -125,6 +125,23 @@ cudaError_t occupancy_resample(int dtype, bool sampled, int* blocks_per_sm);
 cudaError_t launch_philox_fill(unsigned long long seed, uint32_t c0, uint32_t c1, uint32_t c2,
                                uint32_t c3, uint32_t* out, size_t n, cudaStream_t s);
 
+// The drafter's LM head fused with its confidence signals (cmsd_lmhead.cu).
+constexpr int kLhRows = 64;      // hidden rows per block of the LM-head GEMM
+struct LmHeadArgs {
+  const uint16_t* hidden;        // bf16 [R][d]
+  const uint16_t* weight;        // bf16 [V][d]
+  int R, d, V;
+  int nct;                       // CTAs per block of kLhRows rows (each owns a run of the vocabulary)
+  float* logits;                 // nullable: f32 [R][V]
+  Partial* part;                 // [ceil(R / kLhRows)][nct][kLhRows] per-CTA row statistics
+  unsigned* err;                 // error word (bit 2: a wait for a load gave up)
+};
+int lmhead_ctas_per_block(int sms, int R, int V);
+// The GEMM + statistics kernel, then the per-row merge (a programmatic
+// dependent on the same stream).  a carries the parameters, the output
+// pointers and a workspace with row_conf [R].
+cudaError_t launch_lmhead(const LmHeadArgs& h, const StreamArgs& a, cudaStream_t s);
+
 // Host-side checks shared by the entry points (cmsd_api.cu).
 int validate_fused(const void* draft_logits, const void* target_logits, const int32_t* draft_tokens,
                    const int32_t* k_row, int B, int K, int V, int dtype, const void* params,

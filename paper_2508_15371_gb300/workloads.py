@@ -276,8 +276,10 @@ def make_lmhead(R=64, d=2048, V=128256, seed=5, exact=False, spiked=0.7):
     Default recipe (a 1B-class drafter's head at a Llama-3-sized vocabulary):
     W[v, j] ~ N(0, 1) / sqrt(d); each hidden state is N(0, 0.7^2) noise, and
     with probability `spiked` also points at a uniform vocabulary row v* with
-    a height a ~ U[0, 12] (h += a W[v*] / |W[v*]|^2), so the logit at v* is
-    raised by about a: a spread from flat to peaked rows, like c1.
+    a height a ~ U[0, 20] (h += a W[v*] / |W[v*]|^2), so the logit at v* is
+    raised by about a: a spread from flat to peaked rows (at V = 128256 the
+    noise logits alone have a maximum near 3 and a sum near 1.6e5, so a
+    spike needs a height of about 12 to hold half the probability).
 
     exact=True: every entry is a multiple of 1/16 (W in [-1/8, 1/8], h in
     [-1/4, 1/4], a spiked row adds W[v*]), so each product is a multiple of
@@ -286,8 +288,8 @@ def make_lmhead(R=64, d=2048, V=128256, seed=5, exact=False, spiked=0.7):
     """
     rng = np.random.default_rng(np.random.SeedSequence([seed, R, d, V, int(exact)]))
     if exact:
-        w32 = rng.integers(-2, 3, size=(V, d)).astype(np.float32) / 16.0
-        h32 = rng.integers(-2, 3, size=(R, d)).astype(np.float32) / 16.0
+        w32 = rng.integers(-2, 3, size=(V, d), dtype=np.int8).astype(np.float32) / np.float32(16.0)
+        h32 = rng.integers(-2, 3, size=(R, d), dtype=np.int8).astype(np.float32) / np.float32(16.0)
     else:
         w32 = (rng.standard_normal((V, d), dtype=np.float32) / np.float32(np.sqrt(d))).astype(np.float32)
         h32 = (0.7 * rng.standard_normal((R, d), dtype=np.float32)).astype(np.float32)
@@ -301,11 +303,11 @@ def make_lmhead(R=64, d=2048, V=128256, seed=5, exact=False, spiked=0.7):
             if exact:
                 h32[r] += wq[v]
             else:
-                a = rng.uniform(0.0, 12.0)
+                a = rng.uniform(0.0, 20.0)
                 h32[r] += np.float32(a) * wq[v] / np.float32(np.dot(wq[v], wq[v]))
     hb = f32_to_bf16_bits(h32)
     note = ("entries are multiples of 1/16 (float32 dot products exact)" if exact else
-            "W ~ N(0,1)/sqrt(d); h ~ N(0,0.7^2) plus a spike of height U[0,12] towards a uniform token "
+            "W ~ N(0,1)/sqrt(d); h ~ N(0,0.7^2) plus a spike of height U[0,20] towards a uniform token "
             "on %.0f%% of rows" % (100 * spiked))
     return LMHeadWorkload("lmhead", R, d, V, seed, hb, wb, spike, note)
 
