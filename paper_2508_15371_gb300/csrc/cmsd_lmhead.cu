@@ -4,27 +4,26 @@
 // The paper's estimator sits on the drafter's output logits (Sec. I), the
 // product z = h W^T of the drafter's last hidden state with its LM-head
 // weight, and reads from each logit row the entropy, logit margin and softmax
-// margin of Sec. III.B(1).  Here the product runs on the tensor cores
-// (mma.sync m16n8k16, bf16 in, fp32 accumulation; 8 warps, each 64 rows x 32
-// vocabulary entries) and each finished 64 x 256 tile of logits is folded, in
-// the GEMM's epilogue, into per-row running
-// statistics: running maximum and its first index, second largest logit, and
-// compensated sums of e^(z - ref) and e^(z - ref)(z - ref) log2 e against a
-// lazily moved exponent reference (the same arithmetic as the logits pass).
-// The logits never reach HBM unless the caller asks for them.  A second small
-// kernel merges the per-CTA statistics of each row and computes H, margin, C
-// and the log-sum-exp with the logits pass's row arithmetic.
+// margin of Sec. III.B(1).  Here the product runs on the 5th-generation
+// tensor cores (tcgen05.mma, bf16 in, fp32 accumulators in tensor memory) and
+// each finished tile of 128 vocabulary entries x 64 hidden rows is folded, in
+// the GEMM's epilogue, into per-row running statistics: running maximum and
+// its first index, second largest logit, and compensated sums of e^(z - ref)
+// and e^(z - ref)(z - ref) log2 e against a lazily moved exponent reference
+// (the same arithmetic as the logits pass).  The logits never reach HBM
+// unless the caller asks for them.  A second small kernel merges the per-CTA
+// statistics of each row and computes H, margin, C and the log-sum-exp with
+// the logits pass's row arithmetic.
 //
 // Layout: hidden [R][d] and weight [V][d] row-major bf16 (the usual
 // [out][in] layout of a linear layer's weight), d a multiple of 64.  Each CTA
 // owns a contiguous run of the vocabulary for one block of 64 hidden rows and
 // streams its weight rows once through a ring of shared-memory stages filled
 // by 2D tensor-memory-access (TMA) loads: per stage one box of 64 hidden
-// dimensions x 64 hidden rows and one of 64 x 256 weight rows, with the
-// 128-byte swizzle (16-byte chunk c of row r lands at chunk c ^ (r mod 8)), so
-// that ldmatrix reads are free of bank conflicts; rows past R or V arrive as
-// zeros.  The hidden block is re-read from L2 for every tile.  (cp.async
-// loads of the same stages held the weight stream near 3.7 TB/s.)
+// dimensions x 128 weight rows (the MMA's A) and one of 64 x 64 hidden rows
+// (its B), both with the 128-byte swizzle that the MMA's shared-memory
+// descriptors name; rows past R or V arrive as zeros.  The hidden block is
+// re-read from L2 for every tile.
 #include <cuda.h>
 
 #include <mutex>
@@ -34,51 +33,7 @@
 namespace cmsd {
 namespace {
 
-#ifndef CMSD_LH_WARPS
-#define CMSD_LH_WARPS 8
-#endif
-#ifndef CMSD_LH_WARP_COLS
-#define CMSD_LH_WARP_COLS 32
-#endif
-#ifndef CMSD_LH_STAGES
-#define CMSD_LH_STAGES 3
-#endif
-constexpr int kLhWarps = CMSD_LH_WARPS;
-constexpr int kLhWarpCols = CMSD_LH_WARP_COLS;      // vocabulary entries per warp and tile (multiple of 16)
-constexpr int kLhNT = kLhWarpCols / 8;              // n8 tiles per warp
-constexpr int kLhThreads = 32 * kLhWarps;
-constexpr int kLhCols = kLhWarps * kLhWarpCols;     // vocabulary entries per tile
-#ifndef CMSD_LH_DEPTH
-#define CMSD_LH_DEPTH 64
-#endif
-constexpr int kLhDepth = CMSD_LH_DEPTH;             // hidden dimensions per stage (a multiple of 64)
-constexpr int kLhChunks = kLhDepth / 8;             // 16-byte chunks per row of a stage
-constexpr int kLhKs = kLhDepth / 16;                // k16 steps per stage
-constexpr int kLhStages = CMSD_LH_STAGES;
-constexpr int kLhAStage = kLhRows * kLhDepth * 2;   // 8 KB
-constexpr int kLhBStage = kLhCols * kLhDepth * 2;
-constexpr int kLhCPitch = kLhCols + 4;              // floats per row of the epilogue tile
-constexpr int kLhRowThreads = kLhThreads / kLhRows; // threads that fold one row of a tile
-constexpr int kLhFold = kLhCols / kLhRowThreads;    // logits each of them folds per tile
-constexpr size_t kLhStageBytes = (size_t)kLhStages * (kLhAStage + kLhBStage);
-constexpr size_t kLhSmem = 1024 + kLhStageBytes + (size_t)kLhRows * kLhCPitch * 4 + 8 * kLhStages;
-static_assert(kLhWarpCols % 16 == 0 && kLhFold % 32 == 0 && kLhThreads % kLhRows == 0, "tile shape");
-static_assert((kLhRows * kLhChunks) % kLhThreads == 0 && (kLhCols * kLhChunks) % kLhThreads == 0, "stage copy split");
-static_assert(kLhDepth == 64, "one TMA box (128 bytes, the swizzle span) per row and stage");
-static_assert(kLhCols <= 256, "TMA box height");
-static_assert(kLhSmem <= 227 * 1024, "shared memory");
-#ifndef CMSD_LH_CTAS_PER_SM
-#define CMSD_LH_CTAS_PER_SM 1
-#endif
-constexpr int kLhCtasPerSm = CMSD_LH_CTAS_PER_SM;
 constexpr int kMergeRowsPerCta = 8;                 // one warp per row
-
-// Byte offset of 16-byte chunk `ch` of row `row` in a stage whose rows are
-// 2 kLhDepth bytes: chunks are XOR-swizzled by the row's low 3 bits, so the 8
-// rows an ldmatrix phase reads fall on 8 different bank groups.
-__device__ __forceinline__ uint32_t swz(int row, int ch) {
-  return (uint32_t)(row * (2 * kLhDepth) + ((ch ^ (row & 7)) << 4));
-}
 
 // ---- shared-memory barriers and 2D TMA loads -----------------------------------
 __device__ __forceinline__ unsigned long long lh_ns() {
@@ -120,21 +75,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
           "r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
       : "memory");
-}
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(addr));
-}
-
-// c += a b for one 16x8 tile, a 16x16 (row-major fragments), b 16x8 (column fragments)
-__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
 // The vocabulary run of CTA `cta` of a row block: nct near-equal runs of
@@ -187,148 +127,234 @@ __device__ __forceinline__ void fold32(DLane& st, const float* z_src, int v0, in
   kahan(st.t, st.ct, lo32f(ts) + hi32f(ts));
 }
 
-__global__ void __launch_bounds__(kLhThreads, kLhCtasPerSm) lmhead_gemm_kernel(const LmHeadArgs h,
-                                                                    const __grid_constant__ CUtensorMap tmap_h,
-                                                                    const __grid_constant__ CUtensorMap tmap_w) {
-  extern __shared__ __align__(1024) unsigned char lh_smem_raw[];
+// ===========================================================================
+// tcgen05 variant: the product on the 5th-generation tensor cores
+// ===========================================================================
+//
+// One CTA of 192 threads per SM:
+//   warp 0      lane 0 issues the TMA loads of each stage (weight box 64 x 128
+//               rows = the MMA's A, hidden box 64 x 64 rows = its B);
+//   warp 1      allocates TMEM (two 64-column fp32 accumulators), and lane 0
+//               issues tcgen05.mma (M = 128 vocabulary entries, N = 64 hidden
+//               rows, K = 16 per instruction) and the commits;
+//   warps 2..5  the epilogue: warp w reads TMEM lanes 32 (w mod 4) .. (one
+//               vocabulary entry per thread, 64 logits: one per hidden row),
+//               transposes the tile through shared memory and folds it into
+//               the per-row statistics (each thread: one hidden row, one half
+//               of the 128 entries).
+// Barriers: full[s] / empty[s] per stage (TMA -> MMA -> TMA), tfull[b] /
+// tempty[b] per accumulator (MMA -> epilogue -> MMA).  Every wait is bounded;
+// TMEM is released after the last commit and the last load have completed.
+constexpr int kTcM = 128;                           // vocabulary entries per tile (MMA M)
+constexpr int kTcN = kLhRows;                       // hidden rows per block (MMA N)
+constexpr int kTcStages = 6;
+constexpr int kTcAStage = kTcM * 128;               // 16 KB: 128 rows x 64 bf16
+constexpr int kTcBStage = kTcN * 128;               // 8 KB
+constexpr int kTcThreads = 192;
+constexpr int kTcCols = 2 * kTcN;                   // TMEM columns: two accumulators
+constexpr int kTcCPitch = kTcM + 4;                 // floats per row of the transposed tile
+constexpr size_t kTcStageBytes = (size_t)kTcStages * (kTcAStage + kTcBStage);
+constexpr size_t kTcSmem = 1024 + kTcStageBytes + (size_t)kTcN * kTcCPitch * 4 + 8 * (2 * kTcStages + 4) + 16;
+static_assert(kTcSmem <= 227 * 1024, "shared memory");
+
+// Shared-memory matrix descriptor of a K-major tile with 128-byte rows and the
+// 128-byte swizzle: start address, leading offset (unused for this layout),
+// stride between 8-row groups = 1024 bytes, descriptor version 1, layout
+// SWIZZLE_128B.
+__device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+constexpr uint32_t kTcIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kTcN >> 3) << 17) |
+                              ((uint32_t)(kTcM >> 4) << 24);
+
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(kTcIdesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+// 32 lanes x 64 columns of fp32 from TMEM: thread i gets lane (taddr lane + i), columns c .. c + 63
+__device__ __forceinline__ void tc_ld64(uint32_t taddr, float (&v)[64]) {
+  uint32_t r[64];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,"
+      "%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%64];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+        "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]),
+        "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]),
+        "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "r"(taddr)
+      : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int k = 0; k < 64; ++k) v[k] = __uint_as_float(r[k]);
+}
+// named barrier among the 128 epilogue threads (barrier 0 is __syncthreads)
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+__global__ void __launch_bounds__(kTcThreads, 1) lmhead_tc_kernel(const LmHeadArgs h,
+                                                                 const __grid_constant__ CUtensorMap tmap_h,
+                                                                 const __grid_constant__ CUtensorMap tmap_w) {
+  extern __shared__ __align__(1024) unsigned char tc_smem_raw[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int rb = blockIdx.x / h.nct, cta = blockIdx.x - rb * h.nct;
-  // the merge kernel may be scheduled now; it waits for this grid before reading
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   int v0, v1;
   cta_run(h.V, h.nct, cta, v0, v1);
-  const int ntiles = v1 > v0 ? (v1 - v0 + kLhCols - 1) / kLhCols : 0;
-  const int nkc = h.d / kLhDepth;
-  const int G = ntiles * nkc;                      // stages of this CTA
-  const int row0 = rb * kLhRows;
-  // the swizzled TMA boxes want 1024-byte aligned destinations
-  const uint32_t raw = smem_u32(lh_smem_raw);
+  const int ntiles = v1 > v0 ? (v1 - v0 + kTcM - 1) / kTcM : 0;
+  const int nkc = h.d / 64;
+  const int G = ntiles * nkc;
+  const int row0 = rb * kTcN;
+
+  const uint32_t raw = smem_u32(tc_smem_raw);
   const uint32_t pad = ((raw + 1023u) & ~1023u) - raw;
-  unsigned char* lh_smem = lh_smem_raw + pad;
-  const uint32_t sA = raw + pad, sB = sA + kLhStages * kLhAStage;
-  float* sC = reinterpret_cast<float*>(lh_smem + kLhStageBytes);
-  const uint32_t sBar = smem_u32(lh_smem + kLhStageBytes + (size_t)kLhRows * kLhCPitch * 4);
+  unsigned char* sm = tc_smem_raw + pad;
+  const uint32_t sA = raw + pad, sB = sA + kTcStages * kTcAStage;
+  float* sC = reinterpret_cast<float*>(sm + kTcStageBytes);
+  const uint32_t bars = smem_u32(sm + kTcStageBytes + (size_t)kTcN * kTcCPitch * 4);
+  const uint32_t full = bars, empty = bars + 8 * kTcStages;
+  const uint32_t tfull = bars + 16 * kTcStages, tempty = tfull + 16;
+  uint32_t* s_taddr = reinterpret_cast<uint32_t*>(sm + kTcStageBytes + (size_t)kTcN * kTcCPitch * 4 +
+                                                  8 * (2 * kTcStages + 4));
   if (tid == 0) {
-#pragma unroll
-    for (int k = 0; k < kLhStages; ++k) mbar_init(sBar + 8 * k, 1);
+    for (int k = 0; k < kTcStages; ++k) {
+      mbar_init(full + 8 * k, 1);
+      mbar_init(empty + 8 * k, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull + 8 * b, 1);
+      mbar_init(tempty + 8 * b, 128);
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(s_taddr)),
+                 "r"(kTcCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
   __syncthreads();
-  bool ok_waits = true;
+  tc_fence_after();
+  const uint32_t tbase = *s_taddr;
+  bool ok = true;
 
-  // stage g: hidden dimensions [64 kc, 64 kc + 64) of tile t = g / nkc; one
-  // thread arms the stage's barrier and issues both boxes
-  auto load = [&](int g) {
-    const int t = g / nkc, kc = g - t * nkc;
-    const int slot = g % kLhStages;
-    const uint32_t bar = sBar + 8 * slot;
-    mbar_arrive_tx(bar, kLhAStage + kLhBStage);
-    tma_load_2d(sA + slot * kLhAStage, &tmap_h, kc * kLhDepth, row0, bar);
-    tma_load_2d(sB + slot * kLhBStage, &tmap_w, kc * kLhDepth, v0 + t * kLhCols, bar);
-  };
-
-  DLane st;
-  dlane_init(st);
-  float acc[4][kLhNT][4];
-#pragma unroll
-  for (int mt = 0; mt < 4; ++mt)
-#pragma unroll
-    for (int nt = 0; nt < kLhNT; ++nt)
-#pragma unroll
-      for (int k = 0; k < 4; ++k) acc[mt][nt][k] = 0.f;
-
-  if (tid == 0) {
-#pragma unroll
-    for (int s = 0; s < kLhStages - 1; ++s)
-      if (s < G) load(s);
-  }
-  const int j8 = lane >> 3, r8 = lane & 7;
-  for (int g = 0; g < G; ++g) {
-    __syncthreads();                               // every warp is done with stage g - 1 ...
-    if (tid == 0 && g + kLhStages - 1 < G) load(g + kLhStages - 1);   // ... so its slot is refilled
-    const int slot = g % kLhStages;
-    if (ok_waits) ok_waits = mbar_wait(sBar + 8 * slot, (uint32_t)((g / kLhStages) & 1));
-    const uint32_t a_st = sA + slot * kLhAStage, b_st = sB + slot * kLhBStage;
-    // fragments double-buffered: k16 step ks + 1 is read from shared memory
-    // while step ks multiplies
-    uint32_t af[2][4][4], bf[2][kLhNT / 2][4];
-    auto frags = [&](int ks, int buf) {
-#pragma unroll
-      for (int mt = 0; mt < 4; ++mt)
-        ldsm_x4(a_st + swz(mt * 16 + (j8 & 1) * 8 + r8, ks * 2 + (j8 >> 1)), af[buf][mt]);
-#pragma unroll
-      for (int np = 0; np < kLhNT / 2; ++np)      // two n8 tiles per ldmatrix
-        ldsm_x4(b_st + swz(warp * kLhWarpCols + np * 16 + (j8 >> 1) * 8 + r8, ks * 2 + (j8 & 1)), bf[buf][np]);
-    };
-    frags(0, 0);
-#pragma unroll
-    for (int ks = 0; ks < kLhKs; ++ks) {
-      if (ks + 1 < kLhKs) frags(ks + 1, (ks + 1) & 1);
-#pragma unroll
-      for (int mt = 0; mt < 4; ++mt)
-#pragma unroll
-        for (int np = 0; np < kLhNT / 2; ++np) {
-          mma_bf16(acc[mt][2 * np], af[ks & 1][mt], bf[ks & 1][np][0], bf[ks & 1][np][1]);
-          mma_bf16(acc[mt][2 * np + 1], af[ks & 1][mt], bf[ks & 1][np][2], bf[ks & 1][np][3]);
-        }
-    }
-    if ((g + 1) % nkc == 0) {
-      // tile t complete: accumulators -> shared tile -> each thread folds
-      // kLhFold logits of one row (row tid / kLhRowThreads)
-      const int t = g / nkc;
-      const int gq = lane >> 2, tq = lane & 3;
-#pragma unroll
-      for (int mt = 0; mt < 4; ++mt)
-#pragma unroll
-        for (int nt = 0; nt < kLhNT; ++nt) {
-          const int r = mt * 16 + gq, c = warp * kLhWarpCols + nt * 8 + 2 * tq;
-          *reinterpret_cast<float2*>(sC + r * kLhCPitch + c) = make_float2(acc[mt][nt][0], acc[mt][nt][1]);
-          *reinterpret_cast<float2*>(sC + (r + 8) * kLhCPitch + c) = make_float2(acc[mt][nt][2], acc[mt][nt][3]);
-#pragma unroll
-          for (int k = 0; k < 4; ++k) acc[mt][nt][k] = 0.f;
-        }
-      __syncthreads();
-      const int row = tid / kLhRowThreads, qt = tid % kLhRowThreads;
-      const int vq = v0 + t * kLhCols + qt * kLhFold;
-      const float* zs = sC + row * kLhCPitch + qt * kLhFold;
-#pragma unroll 1
-      for (int c = 0; c < kLhFold; c += 32) fold32(st, zs + c, vq + c, v1);
-      if (h.logits && row0 + row < h.R) {
-        float* dst = h.logits + (size_t)(row0 + row) * h.V;
-        for (int k = 0; k < kLhFold && vq + k < v1; ++k) dst[vq + k] = zs[k];
+  if (warp == 0) {
+    // ---- producer ----------------------------------------------------------
+    if (lane == 0) {
+      for (int g = 0; g < G; ++g) {
+        const int slot = g % kTcStages;
+        if (g >= kTcStages && ok) ok = mbar_wait(empty + 8 * slot, (uint32_t)((g / kTcStages - 1) & 1));
+        const int t = g / nkc, kc = g - t * nkc;
+        mbar_arrive_tx(full + 8 * slot, kTcAStage + kTcBStage);
+        tma_load_2d(sA + slot * kTcAStage, &tmap_w, kc * 64, v0 + t * kTcM, full + 8 * slot);
+        tma_load_2d(sB + slot * kTcBStage, &tmap_h, kc * 64, row0, full + 8 * slot);
       }
-      // the tile is rewritten only after the next tile's stages, each of
-      // which starts with a barrier
+    }
+  } else if (warp == 1) {
+    // ---- MMA issuer --------------------------------------------------------
+    if (lane == 0) {
+      for (int t = 0; t < ntiles; ++t) {
+        const int b = t & 1;
+        if (t >= 2 && ok) ok = mbar_wait(tempty + 8 * b, (uint32_t)((t / 2 - 1) & 1));
+        tc_fence_after();
+        const uint32_t d = tbase + (uint32_t)(b * kTcN);
+        for (int kc = 0; kc < nkc; ++kc) {
+          const int g = t * nkc + kc, slot = g % kTcStages;
+          if (ok) ok = mbar_wait(full + 8 * slot, (uint32_t)((g / kTcStages) & 1));
+          tc_fence_after();
+          const uint64_t ad = umma_desc_sw128(sA + slot * kTcAStage);
+          const uint64_t bd = umma_desc_sw128(sB + slot * kTcBStage);
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks)          // K = 16 per instruction: 32 bytes along the row
+            tc_mma(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), (kc | ks) != 0);
+          tc_commit(empty + 8 * slot);             // the stage may be refilled once these MMAs are done
+        }
+        tc_commit(tfull + 8 * b);                  // the accumulator is complete
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---- epilogue: warps 2..5 ------------------------------------------------
+    const int e = tid - 64;                        // 0 .. 127
+    const int q = warp & 3;                        // TMEM lane quarter this warp may read
+    const int m = q * 32 + lane;                   // the vocabulary entry (TMEM lane) this thread reads
+    const int jrow = e >> 1, half = e & 1;         // the hidden row and half-tile this thread folds
+    DLane st;
+    dlane_init(st);
+    for (int t = 0; t < ntiles; ++t) {
+      const int b = t & 1;
+      if (ok) ok = mbar_wait(tfull + 8 * b, (uint32_t)((t / 2) & 1));
+      tc_fence_after();
+      float v[64];
+      tc_ld64(tbase + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * kTcN), v);
+      tc_fence_before();
+      mbar_arrive(tempty + 8 * b);                 // this lane of the accumulator has been read
+      // transpose: row j of the tile holds hidden row j's logits over the 128 entries
+#pragma unroll
+      for (int j = 0; j < kTcN; ++j) sC[j * kTcCPitch + m] = v[j];
+      epi_bar();
+      const int vq = v0 + t * kTcM + half * 64;
+      const float* zs = sC + jrow * kTcCPitch + half * 64;
+      fold32(st, zs, vq, v1);
+      fold32(st, zs + 32, vq + 32, v1);
+      if (h.logits && row0 + jrow < h.R) {
+        float* dst = h.logits + (size_t)(row0 + jrow) * h.V;
+        for (int k = 0; k < 64 && vq + k < v1; ++k) dst[vq + k] = zs[k];
+      }
+      epi_bar();                                   // the tile is rewritten by the next iteration
+    }
+    float s, t2;
+    d_final(st, s, t2);
+    DRed x{d_mexp(st), s, t2, st.f2, st.pos};
+    DRed y;
+    y.m = __shfl_xor_sync(kFull, x.m, 1);
+    y.s = __shfl_xor_sync(kFull, x.s, 1);
+    y.t2 = __shfl_xor_sync(kFull, x.t2, 1);
+    y.top2 = __shfl_xor_sync(kFull, x.top2, 1);
+    y.idx = __shfl_xor_sync(kFull, x.idx, 1);
+    fold_d(x, y);
+    if (half == 0) {
+      Partial p;
+      p.d_m = x.m; p.d_s = x.s; p.d_t2 = x.t2; p.d_top2 = x.top2; p.d_idx = x.idx;
+      p.t_m = 0.f; p.t_s = 0.f; p.t_idx = 0; p.t_cnt = 0;
+      p.pad[0] = p.pad[1] = p.pad[2] = 0;
+      h.part[((size_t)rb * h.nct + cta) * kLhRows + jrow] = p;
     }
   }
-  if (!ok_waits) atomicOr(h.err, 4u);
-  // before the CTA exits, no box may still be in flight into its shared memory
-  if (tid == 0) {
-    for (int g = (G > kLhStages ? G - kLhStages : 0); g < G; ++g)
-      if (!mbar_wait(sBar + 8 * (g % kLhStages), (uint32_t)((g / kLhStages) & 1))) atomicOr(h.err, 4u);
+  if (!ok) atomicOr(h.err, 4u);
+  // teardown: the MMA issuer's last commit covers every MMA of the CTA; then
+  // every thread is past its last TMEM access and TMEM is released
+  if (warp == 1 && lane == 0 && ntiles > 0) {
+    const int t = ntiles - 1;
+    if (!mbar_wait(tfull + 8 * (t & 1), (uint32_t)((t / 2) & 1))) atomicOr(h.err, 4u);
   }
-
-  // the row's kLhRowThreads runs (adjacent lanes), then one partial per (row, CTA)
-  float s, t2;
-  d_final(st, s, t2);
-  DRed x{d_mexp(st), s, t2, st.f2, st.pos};
-#pragma unroll
-  for (int o = 1; o < kLhRowThreads; o <<= 1) {
-    DRed y;
-    y.m = __shfl_xor_sync(kFull, x.m, o);
-    y.s = __shfl_xor_sync(kFull, x.s, o);
-    y.t2 = __shfl_xor_sync(kFull, x.t2, o);
-    y.top2 = __shfl_xor_sync(kFull, x.top2, o);
-    y.idx = __shfl_xor_sync(kFull, x.idx, o);
-    fold_d(x, y);
+  if (warp == 0 && lane == 0) {                    // no TMA box still in flight into this CTA
+    for (int g = (G > kTcStages ? G - kTcStages : 0); g < G; ++g)
+      if (!mbar_wait(full + 8 * (g % kTcStages), (uint32_t)((g / kTcStages) & 1))) atomicOr(h.err, 4u);
   }
-  if (tid % kLhRowThreads == 0) {
-    Partial p;
-    p.d_m = x.m; p.d_s = x.s; p.d_t2 = x.t2; p.d_top2 = x.top2; p.d_idx = x.idx;
-    p.t_m = 0.f; p.t_s = 0.f; p.t_idx = 0; p.t_cnt = 0;
-    p.pad[0] = p.pad[1] = p.pad[2] = 0;
-    h.part[((size_t)rb * h.nct + cta) * kLhRows + tid / kLhRowThreads] = p;
-  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tbase), "r"(kTcCols) : "memory");
 }
 
 // One warp per hidden row: fold the row's per-CTA partials, then the row's
@@ -367,7 +393,7 @@ __global__ void __launch_bounds__(32 * kMergeRowsPerCta) lmhead_merge_kernel(con
 
 int lmhead_ctas_per_block(int sms, int R, int V) {
   const int nrb = (R + kLhRows - 1) / kLhRows;
-  int nct = sms * kLhCtasPerSm / (nrb > 0 ? nrb : 1);
+  int nct = sms / (nrb > 0 ? nrb : 1);
   const int n8 = (V + 7) / 8;
   if (nct > n8) nct = n8;
   return nct < 1 ? 1 : nct;
@@ -399,7 +425,7 @@ bool encode_rows(CUtensorMap* m, const void* base, int d, int rows, int box_rows
   if (!fn) return false;
   const cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
   const cuuint64_t strides[1] = {(cuuint64_t)d * 2};
-  const cuuint32_t box[2] = {(cuuint32_t)kLhDepth, (cuuint32_t)box_rows};
+  const cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -413,16 +439,16 @@ cudaError_t launch_lmhead(const LmHeadArgs& h, const StreamArgs& a, cudaStream_t
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   CUtensorMap tmap_h, tmap_w;
-  if (!encode_rows(&tmap_h, h.hidden, h.d, h.R, kLhRows) || !encode_rows(&tmap_w, h.weight, h.d, h.V, kLhCols))
+  if (!encode_rows(&tmap_h, h.hidden, h.d, h.R, kTcN) || !encode_rows(&tmap_w, h.weight, h.d, h.V, kTcM))
     return cudaErrorInvalidValue;
   const unsigned long long bit = 1ull << (dev & 63);
   if (!(__atomic_load_n(&done, __ATOMIC_ACQUIRE) & bit)) {
-    e = cudaFuncSetAttribute(lmhead_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kLhSmem);
+    e = cudaFuncSetAttribute(lmhead_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTcSmem);
     if (e != cudaSuccess) return e;
     __atomic_fetch_or(&done, bit, __ATOMIC_ACQ_REL);
   }
   const int nrb = (h.R + kLhRows - 1) / kLhRows;
-  lmhead_gemm_kernel<<<nrb * h.nct, kLhThreads, kLhSmem, s>>>(h, tmap_h, tmap_w);
+  lmhead_tc_kernel<<<nrb * h.nct, kTcThreads, kTcSmem, s>>>(h, tmap_h, tmap_w);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
