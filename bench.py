@@ -57,10 +57,22 @@ def peaks():
 KERNEL_SOURCES = ("cmsd_stream_impl.cuh", "cmsd_device.cuh", "cmsd_internal.h")
 
 
-def kernel_sources_sha():
+def measured_peaks():
+    """MEASURED_PEAKS.json as a dict ({} when it is absent)."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f)
+    except Exception:
+        return {}
+
+
+LMHEAD_SOURCES = ("cmsd_lmhead.cu", "cmsd_stream_impl.cuh", "cmsd_device.cuh", "cmsd_internal.h")
+
+
+def kernel_sources_sha(sources=None):
     import hashlib
     h = hashlib.sha256()
-    for n in KERNEL_SOURCES:
+    for n in (KERNEL_SOURCES if sources is None else sources):
         with open(os.path.join(ROOT, "paper_2508_15371_gb300", "csrc", n), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
@@ -405,6 +417,99 @@ def bench_workload(cmsd, torch, dev, name, rule, steps, peak, nsets=1, graph_lat
     return res
 
 
+def lmhead_traffic():
+    """Per-launch DRAM bytes of the LM-head GEMM kernel from the committed ncu
+    summary; None when its sources changed since it was captured."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            for d in json.load(f):
+                if d.get("workload") == "lmhead" and \
+                        d.get("sources_sha256_16") == kernel_sources_sha(LMHEAD_SOURCES):
+                    return d.get("bytes_per_launch")
+    except Exception:
+        pass
+    return None
+
+
+def lmhead_report(cmsd, torch, hbm_peak, R=64, d=2048, V=128256, calls=100):
+    """The drafter's LM head fused with the confidence signals
+    (cmsd_lmhead_confidence): R hidden rows of a d-wide drafter through a
+    [V, d] bf16 head.  Timed with CUDA events over `calls` back-to-back calls
+    (the 525 MB weight is larger than L2); beside it, the same result unfused:
+    a cuBLAS bf16 GEMM (torch.matmul) writing the logits, then
+    cmsd_confidence over them.  Parity: the oracle on 8 of the rows."""
+    from paper_2508_15371_gb300 import workloads as W
+    w = W.make_lmhead(R=R, d=d, V=V, seed=7)
+    h = torch.from_numpy(w.hidden.view(np.int16)).cuda()
+    wt = torch.from_numpy(w.weight.view(np.int16)).cuda()
+    p = cmsd.params(1)
+    ws = cmsd.lmhead_workspace(R, d, V)
+    out = {n: torch.empty(R, dtype=torch.float32, device="cuda") for n in ("H", "margin", "conf", "lse")}
+    out["argmax"] = torch.empty(R, dtype=torch.int32, device="cuda")
+    hb, wb = h.view(torch.bfloat16), wt.view(torch.bfloat16)
+    lg = torch.empty((R, V), dtype=torch.bfloat16, device="cuda")
+    cws = cmsd.workspace(R, 1, V)
+    co = {n: torch.empty((R, 1), dtype=torch.float32, device="cuda") for n in ("H", "margin", "conf", "lse")}
+    co["argmax"] = torch.empty((R, 1), dtype=torch.int32, device="cuda")
+    co["k_next"] = torch.empty(R, dtype=torch.int32, device="cuda")
+
+    def fused():
+        cmsd.lmhead_confidence(h, wt, p=p, out=out, ws=ws)
+
+    def gemm():
+        torch.matmul(hb, wb.t(), out=lg)
+
+    def unfused():
+        gemm()
+        cmsd.confidence(lg.view(R, 1, V), p=p, out=co, ws=cws)
+
+    def timed(fn):
+        for _ in range(5):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(calls):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / calls
+
+    ms_f, ms_g, ms_u = timed(fused), timed(gemm), timed(unfused)
+    g = {k: v.cpu().numpy() for k, v in out.items()}
+    import oracle as O
+    rows = np.arange(0, R, max(1, R // 8))
+    P = O.Params(lam=tuple(p.lam), beta_sig=p.beta_sig)
+    o = O.lm_head_confidence(w.hidden[rows], w.weight, P)
+    habs = np.abs(O.bf16_bits_to_f64(w.hidden[rows]))
+    eps = d * 2.0 ** -23 * (habs @ np.abs(O.bf16_bits_to_f64(w.weight)).T).max(axis=1)
+    clear = o["margin"] > 2 * eps
+    bytes_ = V * d * 2 + R * d * 2
+    flops = 2.0 * R * d * V
+    achieved = bytes_ / (ms_f * 1e-3) / 1e9
+    tflops = flops / (ms_f * 1e-3) / 1e12
+    tpeak = measured_peaks().get("bf16_tflops")
+    return {
+        "workload": f"R={R} hidden rows, d={d}, V={V}, bf16 hidden states and head weight "
+                    "(a 1B-class drafter's LM head at the Llama-3 vocabulary)",
+        "ms_per_call": ms_f, "rows_per_s": R / (ms_f * 1e-3),
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved / hbm_peak, "traffic": lmhead_traffic(),
+                     "algorithmic_bytes_per_call": bytes_,
+                     "kernel": "lmhead_tc_kernel (tcgen05 GEMM + statistics epilogue) and the row merge"},
+        "tensor": {"achieved_tflops": tflops, "peak_tflops": tpeak, "frac": tflops / tpeak if tpeak else None,
+                   "peak_source": "measured (MEASURED_PEAKS.json bf16_tflops, cuBLAS burst)" if tpeak else None,
+                   "flops_per_call": flops},
+        "unfused_ms": ms_u, "cublas_gemm_only_ms": ms_g, "speedup_vs_unfused": ms_u / ms_f,
+        "parity": {"rows": int(len(rows)),
+                   "argmax_equal": int(np.sum((g["argmax"][rows] == o["argmax"]) & clear)),
+                   "argmax_compared": int(np.sum(clear)),
+                   "max_abs_err": {k: float(np.max(np.abs(g[k][rows] - o[k]))) for k in ("H", "lse", "conf")},
+                   "logit_rounding_bound": float(eps.max())},
+        "timing": f"CUDA events over {calls} back-to-back calls after 5 warm-up calls; weight 525 MB > L2",
+    }
+
+
 def decode_sim_report(cmsd, torch, B=32, K=16, V=32000, iterations=512):
     """Algorithm 1 as a decode loop over device-generated f32 logits (k_next
     of each iteration is the next iteration's k_row), captured in a CUDA
@@ -486,6 +591,9 @@ def run_ours(args):
     if args.only:
         # one workload's device-resident timing, nothing else (for profiling a
         # single configuration's launches)
+        if args.only == "lmhead":
+            print(json.dumps(lmhead_report(cmsd, torch, peak, calls=max(3, args.steps))), flush=True)
+            return 0
         steps = max(3, args.steps)
         size = {"B": args.batch} if args.batch else {}
         print(json.dumps(bench_workload(cmsd, torch, dev, args.only, args.rule, steps, peak, **size)), flush=True)
@@ -637,6 +745,8 @@ def run_ours(args):
         # ---- decode-loop simulation --------------------------------------------
         if not args.no_decode_sim:
             extra["decode_sim"] = decode_sim_report(cmsd, torch)
+        # ---- the drafter's LM head fused with the signals ----------------------
+        extra["lmhead"] = lmhead_report(cmsd, torch, peak)
 
     # ---- CPU oracle baseline, with a live parity check of its sample ---------
     cpu = None
@@ -703,7 +813,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-decode-sim", action="store_true", help="skip the decode-loop simulation report")
     ap.add_argument("--no-extra", action="store_true", help="headline only (no other workloads, no decode loop)")
-    ap.add_argument("--only", choices=["c1", "c2", "c3", "c4"], default=None,
+    ap.add_argument("--only", choices=["c1", "c2", "c3", "c4", "lmhead"], default=None,
                     help="time one workload under --rule and print its object only (for profiling)")
     ap.add_argument("--batch", type=int, default=0, help="with --only: the number of sequences B (default: full)")
     ap.add_argument("--load-window", type=float, default=0.8,
