@@ -159,7 +159,9 @@ int cmsd_confidence(const void* draft_logits, int B, int K, int V, int dtype,
  *   hidden: bf16 [R][d] device, row-major; weight: bf16 [V][d] device,
  *     row-major (the [out][in] layout of a linear layer); both 16-byte
  *     aligned; d a multiple of 64, 64 <= d <= 2^20; 2 <= V; R*V < 2^46;
- *     R == 0 is a valid empty call.  Entries must be finite.
+ *     R == 0 is a valid empty call.  Entries must be finite.  Up to 256
+ *     hidden rows share one pass over the weight (more take one pass per
+ *     256 rows).
  *   z is accumulated in fp32 from exact bf16 products (tensor cores), in an
  *   order that differs from a sequential sum: each logit differs from the
  *   exact dot product by rounding only.

@@ -311,17 +311,18 @@ int validate_fused(const void* draft_logits, const void* target_logits, const in
 namespace {
 struct LmLayout {
   size_t row_conf, part, total;
-  int nct;
+  int nct, nb;
 };
 int lm_layout(int R, int V, LmLayout* L) {
   int sms = 0;
   int rc = device_sms(&sms);
   if (rc) return rc;
   L->nct = lmhead_ctas_per_block(sms, R, V);
-  const size_t nrb = (size_t)(R + kLhRows - 1) / kLhRows;
+  L->nb = lmhead_block_rows(R);
+  const size_t nrb = (size_t)(R + L->nb - 1) / L->nb;
   size_t o = up(sizeof(unsigned));
   L->row_conf = o; o += up((size_t)R * sizeof(unsigned long long));
-  L->part = o; o += up(nrb * (size_t)L->nct * kLhRows * sizeof(Partial));
+  L->part = o; o += up(nrb * (size_t)L->nct * L->nb * sizeof(Partial));
   L->total = o;
   return CMSD_OK;
 }
@@ -401,6 +402,7 @@ int cmsd_lmhead_confidence(const void* hidden, const void* weight, int R, int d,
   h.weight = (const uint16_t*)weight;
   h.R = R; h.d = d; h.V = V;
   h.nct = L.nct;
+  h.nb = L.nb;
   h.logits = logits;
   h.part = (Partial*)(w + L.part);
   h.err = a.ws.err;

@@ -126,16 +126,17 @@ cudaError_t launch_philox_fill(unsigned long long seed, uint32_t c0, uint32_t c1
                                uint32_t c3, uint32_t* out, size_t n, cudaStream_t s);
 
 // The drafter's LM head fused with its confidence signals (cmsd_lmhead.cu).
-constexpr int kLhRows = 64;      // hidden rows per block of the LM-head GEMM
 struct LmHeadArgs {
   const uint16_t* hidden;        // bf16 [R][d]
   const uint16_t* weight;        // bf16 [V][d]
   int R, d, V;
-  int nct;                       // CTAs per block of kLhRows rows (each owns a run of the vocabulary)
+  int nb;                        // hidden rows per block (lmhead_block_rows(R))
+  int nct;                       // CTAs per block (each owns a run of the vocabulary)
   float* logits;                 // nullable: f32 [R][V]
-  Partial* part;                 // [ceil(R / kLhRows)][nct][kLhRows] per-CTA row statistics
+  Partial* part;                 // [ceil(R / nb)][nct][nb] per-CTA row statistics
   unsigned* err;                 // error word (bit 2: a wait for a load gave up)
 };
+int lmhead_block_rows(int R);
 int lmhead_ctas_per_block(int sms, int R, int V);
 // The GEMM + statistics kernel, then the per-row merge (a programmatic
 // dependent on the same stream).  a carries the parameters, the output

@@ -146,16 +146,29 @@ __device__ __forceinline__ void fold32(DLane& st, const float* z_src, int v0, in
 // tempty[b] per accumulator (MMA -> epilogue -> MMA).  Every wait is bounded;
 // TMEM is released after the last commit and the last load have completed.
 constexpr int kTcM = 128;                           // vocabulary entries per tile (MMA M)
-constexpr int kTcN = kLhRows;                       // hidden rows per block (MMA N)
-constexpr int kTcStages = 6;
 constexpr int kTcAStage = kTcM * 128;               // 16 KB: 128 rows x 64 bf16
-constexpr int kTcBStage = kTcN * 128;               // 8 KB
 constexpr int kTcThreads = 192;
-constexpr int kTcCols = 2 * kTcN;                   // TMEM columns: two accumulators
-constexpr int kTcCPitch = kTcM + 4;                 // floats per row of the transposed tile
-constexpr size_t kTcStageBytes = (size_t)kTcStages * (kTcAStage + kTcBStage);
-constexpr size_t kTcSmem = 1024 + kTcStageBytes + (size_t)kTcN * kTcCPitch * 4 + 8 * (2 * kTcStages + 4) + 16;
-static_assert(kTcSmem <= 227 * 1024, "shared memory");
+constexpr int kTcCPitch = kTcM + 4;                 // floats per row of the transposed 64-row chunk
+
+// Shapes for a block of N hidden rows (the MMA's N: 64, 128 or 256).  The
+// accumulators take 2N TMEM columns; the epilogue walks them in chunks of 64
+// columns (hidden rows); the stage count fills the shared memory.
+template <int N>
+struct TcShape {
+  static_assert(N == 64 || N == 128 || N == 256, "block rows");
+  static constexpr int kStages = N == 256 ? 4 : (N == 128 ? 5 : 6);
+  static constexpr int kBStage = N * 128;
+  static constexpr int kCols = 2 * N;
+  static constexpr int kChunks = N / 64;
+  static constexpr size_t kStageBytes = (size_t)kStages * (kTcAStage + kBStage);
+  static constexpr size_t kCBytes = (size_t)64 * kTcCPitch * 4;
+  static constexpr size_t kSmem = 1024 + kStageBytes + kCBytes + 8 * (2 * kStages + 4) + 16;
+  // instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
+  // K-major, N >> 3 at bit 17, M >> 4 at bit 24
+  static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
+                                     ((uint32_t)(kTcM >> 4) << 24);
+  static_assert(kSmem <= 227 * 1024, "shared memory");
+};
 
 // Shared-memory matrix descriptor of a K-major tile with 128-byte rows and the
 // 128-byte swizzle: start address, leading offset (unused for this layout),
@@ -165,16 +178,13 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
   return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
          ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
-// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
-// K-major, N >> 3 at bit 17, M >> 4 at bit 24.
-constexpr uint32_t kTcIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kTcN >> 3) << 17) |
-                              ((uint32_t)(kTcM >> 4) << 24);
 
-__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                       uint32_t accumulate) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(kTcIdesc), "r"(accumulate)
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
@@ -209,9 +219,12 @@ __device__ __forceinline__ void tc_ld64(uint32_t taddr, float (&v)[64]) {
 // named barrier among the 128 epilogue threads (barrier 0 is __syncthreads)
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
+template <int N>
 __global__ void __launch_bounds__(kTcThreads, 1) lmhead_tc_kernel(const LmHeadArgs h,
                                                                  const __grid_constant__ CUtensorMap tmap_h,
                                                                  const __grid_constant__ CUtensorMap tmap_w) {
+  using S = TcShape<N>;
+  constexpr int kStages = S::kStages;
   extern __shared__ __align__(1024) unsigned char tc_smem_raw[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int rb = blockIdx.x / h.nct, cta = blockIdx.x - rb * h.nct;
@@ -221,20 +234,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) lmhead_tc_kernel(const LmHeadAr
   const int ntiles = v1 > v0 ? (v1 - v0 + kTcM - 1) / kTcM : 0;
   const int nkc = h.d / 64;
   const int G = ntiles * nkc;
-  const int row0 = rb * kTcN;
+  const int row0 = rb * N;
 
   const uint32_t raw = smem_u32(tc_smem_raw);
   const uint32_t pad = ((raw + 1023u) & ~1023u) - raw;
   unsigned char* sm = tc_smem_raw + pad;
-  const uint32_t sA = raw + pad, sB = sA + kTcStages * kTcAStage;
-  float* sC = reinterpret_cast<float*>(sm + kTcStageBytes);
-  const uint32_t bars = smem_u32(sm + kTcStageBytes + (size_t)kTcN * kTcCPitch * 4);
-  const uint32_t full = bars, empty = bars + 8 * kTcStages;
-  const uint32_t tfull = bars + 16 * kTcStages, tempty = tfull + 16;
-  uint32_t* s_taddr = reinterpret_cast<uint32_t*>(sm + kTcStageBytes + (size_t)kTcN * kTcCPitch * 4 +
-                                                  8 * (2 * kTcStages + 4));
+  const uint32_t sA = raw + pad, sB = sA + kStages * kTcAStage;
+  float* sC = reinterpret_cast<float*>(sm + S::kStageBytes);
+  const uint32_t bars = smem_u32(sm + S::kStageBytes + S::kCBytes);
+  const uint32_t full = bars, empty = bars + 8 * kStages;
+  const uint32_t tfull = bars + 16 * kStages, tempty = tfull + 16;
+  uint32_t* s_taddr = reinterpret_cast<uint32_t*>(sm + S::kStageBytes + S::kCBytes + 8 * (2 * kStages + 4));
   if (tid == 0) {
-    for (int k = 0; k < kTcStages; ++k) {
+    for (int k = 0; k < kStages; ++k) {
       mbar_init(full + 8 * k, 1);
       mbar_init(empty + 8 * k, 1);
     }
@@ -246,7 +258,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) lmhead_tc_kernel(const LmHeadAr
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(s_taddr)),
-                 "r"(kTcCols)
+                 "r"(S::kCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -260,12 +272,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) lmhead_tc_kernel(const LmHeadAr
     // ---- producer ----------------------------------------------------------
     if (lane == 0) {
       for (int g = 0; g < G; ++g) {
-        const int slot = g % kTcStages;
-        if (g >= kTcStages && ok) ok = mbar_wait(empty + 8 * slot, (uint32_t)((g / kTcStages - 1) & 1));
+        const int slot = g % kStages;
+        if (g >= kStages && ok) ok = mbar_wait(empty + 8 * slot, (uint32_t)((g / kStages - 1) & 1));
         const int t = g / nkc, kc = g - t * nkc;
-        mbar_arrive_tx(full + 8 * slot, kTcAStage + kTcBStage);
+        mbar_arrive_tx(full + 8 * slot, kTcAStage + S::kBStage);
         tma_load_2d(sA + slot * kTcAStage, &tmap_w, kc * 64, v0 + t * kTcM, full + 8 * slot);
-        tma_load_2d(sB + slot * kTcBStage, &tmap_h, kc * 64, row0, full + 8 * slot);
+        tma_load_2d(sB + slot * S::kBStage, &tmap_h, kc * 64, row0, full + 8 * slot);
       }
     }
   } else if (warp == 1) {
@@ -275,16 +287,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) lmhead_tc_kernel(const LmHeadAr
         const int b = t & 1;
         if (t >= 2 && ok) ok = mbar_wait(tempty + 8 * b, (uint32_t)((t / 2 - 1) & 1));
         tc_fence_after();
-        const uint32_t d = tbase + (uint32_t)(b * kTcN);
+        const uint32_t d = tbase + (uint32_t)(b * N);
         for (int kc = 0; kc < nkc; ++kc) {
-          const int g = t * nkc + kc, slot = g % kTcStages;
-          if (ok) ok = mbar_wait(full + 8 * slot, (uint32_t)((g / kTcStages) & 1));
+          const int g = t * nkc + kc, slot = g % kStages;
+          if (ok) ok = mbar_wait(full + 8 * slot, (uint32_t)((g / kStages) & 1));
           tc_fence_after();
           const uint64_t ad = umma_desc_sw128(sA + slot * kTcAStage);
-          const uint64_t bd = umma_desc_sw128(sB + slot * kTcBStage);
+          const uint64_t bd = umma_desc_sw128(sB + slot * S::kBStage);
 #pragma unroll
           for (int ks = 0; ks < 4; ++ks)          // K = 16 per instruction: 32 bytes along the row
-            tc_mma(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), (kc | ks) != 0);
+            tc_mma(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), S::kIdesc, (kc | ks) != 0);
           tc_commit(empty + 8 * slot);             // the stage may be refilled once these MMAs are done
         }
         tc_commit(tfull + 8 * b);                  // the accumulator is complete
@@ -296,47 +308,57 @@ __global__ void __launch_bounds__(kTcThreads, 1) lmhead_tc_kernel(const LmHeadAr
     const int e = tid - 64;                        // 0 .. 127
     const int q = warp & 3;                        // TMEM lane quarter this warp may read
     const int m = q * 32 + lane;                   // the vocabulary entry (TMEM lane) this thread reads
-    const int jrow = e >> 1, half = e & 1;         // the hidden row and half-tile this thread folds
-    DLane st;
-    dlane_init(st);
+    const int jrow = e >> 1, half = e & 1;         // within each 64-row chunk: the row and half-tile it folds
+    DLane st[S::kChunks];
+#pragma unroll
+    for (int c = 0; c < S::kChunks; ++c) dlane_init(st[c]);
     for (int t = 0; t < ntiles; ++t) {
       const int b = t & 1;
       if (ok) ok = mbar_wait(tfull + 8 * b, (uint32_t)((t / 2) & 1));
       tc_fence_after();
-      float v[64];
-      tc_ld64(tbase + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * kTcN), v);
-      tc_fence_before();
-      mbar_arrive(tempty + 8 * b);                 // this lane of the accumulator has been read
-      // transpose: row j of the tile holds hidden row j's logits over the 128 entries
 #pragma unroll
-      for (int j = 0; j < kTcN; ++j) sC[j * kTcCPitch + m] = v[j];
-      epi_bar();
-      const int vq = v0 + t * kTcM + half * 64;
-      const float* zs = sC + jrow * kTcCPitch + half * 64;
-      fold32(st, zs, vq, v1);
-      fold32(st, zs + 32, vq + 32, v1);
-      if (h.logits && row0 + jrow < h.R) {
-        float* dst = h.logits + (size_t)(row0 + jrow) * h.V;
-        for (int k = 0; k < 64 && vq + k < v1; ++k) dst[vq + k] = zs[k];
+      for (int c = 0; c < S::kChunks; ++c) {
+        float v[64];
+        tc_ld64(tbase + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * N + 64 * c), v);
+        if (c == S::kChunks - 1) {
+          tc_fence_before();
+          mbar_arrive(tempty + 8 * b);             // this lane of the accumulator has been read
+        }
+        // transpose: row j of the chunk holds hidden row 64 c + j's logits over the 128 entries
+#pragma unroll
+        for (int j = 0; j < 64; ++j) sC[j * kTcCPitch + m] = v[j];
+        epi_bar();
+        const int vq = v0 + t * kTcM + half * 64;
+        const float* zs = sC + jrow * kTcCPitch + half * 64;
+        fold32(st[c], zs, vq, v1);
+        fold32(st[c], zs + 32, vq + 32, v1);
+        const int grow = row0 + 64 * c + jrow;
+        if (h.logits && grow < h.R) {
+          float* dst = h.logits + (size_t)grow * h.V;
+          for (int k = 0; k < 64 && vq + k < v1; ++k) dst[vq + k] = zs[k];
+        }
+        epi_bar();                                 // the chunk buffer is rewritten next
       }
-      epi_bar();                                   // the tile is rewritten by the next iteration
     }
-    float s, t2;
-    d_final(st, s, t2);
-    DRed x{d_mexp(st), s, t2, st.f2, st.pos};
-    DRed y;
-    y.m = __shfl_xor_sync(kFull, x.m, 1);
-    y.s = __shfl_xor_sync(kFull, x.s, 1);
-    y.t2 = __shfl_xor_sync(kFull, x.t2, 1);
-    y.top2 = __shfl_xor_sync(kFull, x.top2, 1);
-    y.idx = __shfl_xor_sync(kFull, x.idx, 1);
-    fold_d(x, y);
-    if (half == 0) {
-      Partial p;
-      p.d_m = x.m; p.d_s = x.s; p.d_t2 = x.t2; p.d_top2 = x.top2; p.d_idx = x.idx;
-      p.t_m = 0.f; p.t_s = 0.f; p.t_idx = 0; p.t_cnt = 0;
-      p.pad[0] = p.pad[1] = p.pad[2] = 0;
-      h.part[((size_t)rb * h.nct + cta) * kLhRows + jrow] = p;
+#pragma unroll
+    for (int c = 0; c < S::kChunks; ++c) {
+      float s, t2;
+      d_final(st[c], s, t2);
+      DRed x{d_mexp(st[c]), s, t2, st[c].f2, st[c].pos};
+      DRed y;
+      y.m = __shfl_xor_sync(kFull, x.m, 1);
+      y.s = __shfl_xor_sync(kFull, x.s, 1);
+      y.t2 = __shfl_xor_sync(kFull, x.t2, 1);
+      y.top2 = __shfl_xor_sync(kFull, x.top2, 1);
+      y.idx = __shfl_xor_sync(kFull, x.idx, 1);
+      fold_d(x, y);
+      if (half == 0) {
+        Partial p;
+        p.d_m = x.m; p.d_s = x.s; p.d_t2 = x.t2; p.d_top2 = x.top2; p.d_idx = x.idx;
+        p.t_m = 0.f; p.t_s = 0.f; p.t_idx = 0; p.t_cnt = 0;
+        p.pad[0] = p.pad[1] = p.pad[2] = 0;
+        h.part[((size_t)rb * h.nct + cta) * N + 64 * c + jrow] = p;
+      }
     }
   }
   if (!ok) atomicOr(h.err, 4u);
@@ -347,14 +369,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) lmhead_tc_kernel(const LmHeadAr
     if (!mbar_wait(tfull + 8 * (t & 1), (uint32_t)((t / 2) & 1))) atomicOr(h.err, 4u);
   }
   if (warp == 0 && lane == 0) {                    // no TMA box still in flight into this CTA
-    for (int g = (G > kTcStages ? G - kTcStages : 0); g < G; ++g)
-      if (!mbar_wait(full + 8 * (g % kTcStages), (uint32_t)((g / kTcStages) & 1))) atomicOr(h.err, 4u);
+    for (int g = (G > kStages ? G - kStages : 0); g < G; ++g)
+      if (!mbar_wait(full + 8 * (g % kStages), (uint32_t)((g / kStages) & 1))) atomicOr(h.err, 4u);
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   if (warp == 1)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tbase), "r"(kTcCols) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tbase), "r"(S::kCols) : "memory");
 }
 
 // One warp per hidden row: fold the row's per-CTA partials, then the row's
@@ -364,8 +386,8 @@ __global__ void __launch_bounds__(32 * kMergeRowsPerCta) lmhead_merge_kernel(con
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * kMergeRowsPerCta + (threadIdx.x >> 5);
   if (r >= h.R) return;                            // whole warps
-  const int rb = r / kLhRows, row = r - rb * kLhRows;
-  const Partial* base = h.part + (size_t)rb * h.nct * kLhRows + row;
+  const int rb = r / h.nb, row = r - rb * h.nb;
+  const Partial* base = h.part + (size_t)rb * h.nct * h.nb + row;
   DRed m = dred_empty();
   constexpr int kBatch = 8;                        // partials in flight per lane
   for (int k0 = lane; k0 < h.nct; k0 += 32 * kBatch) {
@@ -374,7 +396,7 @@ __global__ void __launch_bounds__(32 * kMergeRowsPerCta) lmhead_merge_kernel(con
     for (int j = 0; j < kBatch; ++j) {
       const int k = k0 + 32 * j;
       if (k < h.nct) {
-        const float4* src = reinterpret_cast<const float4*>(base + (size_t)k * kLhRows);
+        const float4* src = reinterpret_cast<const float4*>(base + (size_t)k * h.nb);
         x0[j] = __ldcg(src);
         x1[j] = __ldcg(src + 1);
       }
@@ -391,8 +413,13 @@ __global__ void __launch_bounds__(32 * kMergeRowsPerCta) lmhead_merge_kernel(con
 
 }  // namespace
 
+// Hidden rows per block: the least of 64, 128, 256 that holds R (more rows
+// than 256 take several blocks, each reading the weight once).
+int lmhead_block_rows(int R) { return R <= 64 ? 64 : (R <= 128 ? 128 : 256); }
+
 int lmhead_ctas_per_block(int sms, int R, int V) {
-  const int nrb = (R + kLhRows - 1) / kLhRows;
+  const int nb = lmhead_block_rows(R);
+  const int nrb = (R + nb - 1) / nb;
   int nct = sms / (nrb > 0 ? nrb : 1);
   const int n8 = (V + 7) / 8;
   if (nct > n8) nct = n8;
@@ -433,23 +460,30 @@ bool encode_rows(CUtensorMap* m, const void* base, int d, int rows, int box_rows
 }
 }  // namespace
 
-cudaError_t launch_lmhead(const LmHeadArgs& h, const StreamArgs& a, cudaStream_t s) {
+template <int N>
+cudaError_t launch_tc(const LmHeadArgs& h, cudaStream_t s) {
   static unsigned long long done = 0ull;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   CUtensorMap tmap_h, tmap_w;
-  if (!encode_rows(&tmap_h, h.hidden, h.d, h.R, kTcN) || !encode_rows(&tmap_w, h.weight, h.d, h.V, kTcM))
+  if (!encode_rows(&tmap_h, h.hidden, h.d, h.R, N) || !encode_rows(&tmap_w, h.weight, h.d, h.V, kTcM))
     return cudaErrorInvalidValue;
   const unsigned long long bit = 1ull << (dev & 63);
   if (!(__atomic_load_n(&done, __ATOMIC_ACQUIRE) & bit)) {
-    e = cudaFuncSetAttribute(lmhead_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTcSmem);
+    e = cudaFuncSetAttribute(lmhead_tc_kernel<N>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)TcShape<N>::kSmem);
     if (e != cudaSuccess) return e;
     __atomic_fetch_or(&done, bit, __ATOMIC_ACQ_REL);
   }
-  const int nrb = (h.R + kLhRows - 1) / kLhRows;
-  lmhead_tc_kernel<<<nrb * h.nct, kTcThreads, kTcSmem, s>>>(h, tmap_h, tmap_w);
-  e = cudaGetLastError();
+  const int nrb = (h.R + N - 1) / N;
+  lmhead_tc_kernel<N><<<nrb * h.nct, kTcThreads, TcShape<N>::kSmem, s>>>(h, tmap_h, tmap_w);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lmhead(const LmHeadArgs& h, const StreamArgs& a, cudaStream_t s) {
+  if (h.nb != lmhead_block_rows(h.R)) return cudaErrorInvalidValue;
+  cudaError_t e = h.nb == 64 ? launch_tc<64>(h, s) : (h.nb == 128 ? launch_tc<128>(h, s) : launch_tc<256>(h, s));
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)((h.R + kMergeRowsPerCta - 1) / kMergeRowsPerCta));

@@ -48,8 +48,10 @@ def _params(cmsd, **kw):
     return p, P
 
 
-@pytest.mark.parametrize("R,d,V", [(5, 256, 1000), (3, 64, 1003), (1, 128, 2), (64, 512, 4096),
-                                   (130, 128, 5000), (7, 192, 129)])
+# R picks the hidden-row block: 64 (R <= 64), 128 (R <= 128), 256 (more; R > 256 takes several blocks)
+@pytest.mark.parametrize("R,d,V", [(5, 256, 1000), (3, 64, 1003), (1, 128, 2), (64, 512, 4096), (7, 192, 129),
+                                   (65, 128, 3000), (128, 256, 2049), (130, 128, 5000), (256, 64, 1500),
+                                   (300, 128, 777)])
 def test_exact_inputs_bit_exact(cmsd, R, d, V):
     w = W.make_lmhead(R=R, d=d, V=V, seed=R + d + V, exact=True)
     p, P = _params(cmsd)
