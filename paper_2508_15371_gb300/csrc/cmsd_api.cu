@@ -247,10 +247,17 @@ int launch(int dtype, int mode, bool sampled, StreamArgs& a, void* ws, size_t ws
   int grid = 0;
   rc = stream_grid(dtype, mode, sampled, second, smem, &grid);
   if (rc) return rc;
-  int g2 = 0;
+  int g2 = 0, nclu = 0;
+  // the sampled rule's residual draw without the bonus row: by group bounds,
+  // one cluster per queued row (up to two per SM pair's worth; more rows loop)
+  const bool bound = second && sampled && !bonus && resample_bound_fits(dtype, a.V);
   if (second) {
     rc = resample_grid(dtype, sampled, &g2);
     if (rc) return rc;
+    int sms = 0;
+    rc = device_sms(&sms);
+    if (rc) return rc;
+    nclu = a.B < 2 * sms ? a.B : 2 * sms;
   }
   a.nwarps = grid * kStreamWarps;
   prof_record(0, s);
@@ -261,7 +268,10 @@ int launch(int dtype, int mode, bool sampled, StreamArgs& a, void* ws, size_t ws
   if (second) {
     StreamArgs b = a;
     b.nwarps = g2 * kResWarps;
-    e = dtype == CMSD_F32 ? launch_resample_f32(sampled, b, g2, s) : launch_resample_bf16(sampled, b, g2, s);
+    if (bound)
+      e = dtype == CMSD_F32 ? launch_resample_bound_f32(b, nclu, s) : launch_resample_bound_bf16(b, nclu, s);
+    else
+      e = dtype == CMSD_F32 ? launch_resample_f32(sampled, b, g2, s) : launch_resample_bf16(sampled, b, g2, s);
     if (e != cudaSuccess) {
       // the streaming kernel has queued rows that no resample kernel will
       // drain: return the queue counters to zero so the workspace stays usable

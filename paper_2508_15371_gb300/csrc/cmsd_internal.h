@@ -119,6 +119,12 @@ cudaError_t launch_stream_bf16(int mode, bool sampled, bool second, const Stream
                                size_t smem, cudaStream_t s);
 cudaError_t launch_resample_f32(bool sampled, const StreamArgs& a, int grid, cudaStream_t s);
 cudaError_t launch_resample_bf16(bool sampled, const StreamArgs& a, int grid, cudaStream_t s);
+// The residual draw by group bounds (sampled rule, no bonus row): clusters
+// of CTAs, one queued row per cluster at a time; resample_bound_fits says
+// whether a row's share fits its shared memory (else resample_kernel).
+cudaError_t launch_resample_bound_f32(const StreamArgs& a, int clusters, cudaStream_t s);
+cudaError_t launch_resample_bound_bf16(const StreamArgs& a, int clusters, cudaStream_t s);
+bool resample_bound_fits(int dtype, int V);
 cudaError_t occupancy_stream(int dtype, int mode, bool sampled, bool second, size_t smem,
                              int* blocks_per_sm);
 cudaError_t occupancy_resample(int dtype, bool sampled, int* blocks_per_sm);

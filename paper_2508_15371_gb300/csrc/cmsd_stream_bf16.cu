@@ -16,6 +16,10 @@ cudaError_t launch_resample_bf16(bool sampled, const StreamArgs& a, int grid, cu
   return launch_resample_t<uint16_t>(sampled, a, grid, s);
 }
 
+cudaError_t launch_resample_bound_bf16(const StreamArgs& a, int clusters, cudaStream_t s) {
+  return launch_resample_bound_t<uint16_t>(a, clusters, s);
+}
+
 cudaError_t occupancy_resample_bf16(bool sampled, int* nb) { return occupancy_resample_t<uint16_t>(sampled, nb); }
 
 }  // namespace cmsd

@@ -11,6 +11,14 @@ cudaError_t launch_resample_f32(bool sampled, const StreamArgs& a, int grid, cud
   return launch_resample_t<float>(sampled, a, grid, s);
 }
 
+cudaError_t launch_resample_bound_f32(const StreamArgs& a, int clusters, cudaStream_t s) {
+  return launch_resample_bound_t<float>(a, clusters, s);
+}
+
+bool resample_bound_fits(int dtype, int V) {
+  return (dtype == 0 ? clu_smem_bytes<float>(V) : clu_smem_bytes<uint16_t>(V)) <= kCluSmemMax;
+}
+
 cudaError_t occupancy_resample(int dtype, bool sampled, int* nb) {
   return dtype == 0 ? occupancy_resample_t<float>(sampled, nb) : occupancy_resample_bf16(sampled, nb);
 }

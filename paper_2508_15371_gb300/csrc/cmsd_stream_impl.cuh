@@ -48,12 +48,15 @@
 // -inf logits (masked vocabulary) are clamped to -2^100 before the drafter
 // arithmetic so that e^(z-m) * (z-m) is 0, not NaN.
 #pragma once
+#include <cooperative_groups.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
 #include "cmsd_device.cuh"
 #include "cmsd_internal.h"
 #include "cmsd_philox.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace cmsd {
 
@@ -1216,8 +1219,9 @@ __device__ __forceinline__ int race_group_entries(uint4 qt, uint4 qd, int gm, in
   const uint32_t sel = (uint32_t)v & 3u;
   const uint32_t word = sel == 0 ? wd.x : sel == 1 ? wd.y : sel == 2 ? wd.z : wd.w;
   const float key = rv > 0.f ? expo(word) / rv : pos_inf();
-  const float km = warp_min(key);
-  const int vm = warp_min_i(key == km ? v : kIntMax);
+  // keys are >= 0 or +inf: their bits order as unsigned integers
+  const float km = __uint_as_float(__reduce_min_sync(kFull, __float_as_uint(key)));
+  const int vm = __reduce_min_sync(kFull, key == km ? v : kIntMax);
   return km != pos_inf() ? vm : -1;
 }
 
@@ -1578,6 +1582,342 @@ __global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_ker
 }
 
 // ---------------------------------------------------------------------------
+// residual draw by group bounds (sampled rule, no bonus row)
+// ---------------------------------------------------------------------------
+//
+// The same two-level race, with the same keys, reading far less.  Since
+// r_v = max(0, p_v - q_v) <= p_v <= p(m_g), m_g the largest target logit of
+// group g, the group's residual mass has the bound
+//   R_g <= Rb_g = kGroup p(m_g) (1 + 2^-16) + 2^-100
+// (the factor covers the rounding of the 32-term sum and of ex2, the floor
+// entries whose p underflows), and its key E_g / R_g >= U_g / Rb_g because
+// E = -log(1 - U) >= U.  A cluster of kCluCtas CTAs takes one queued row, a
+// share of its groups each:
+//   stage   the share of the target row is copied to shared memory (cp.async)
+//           while the share's uniforms are drawn;
+//   bound   m_g and Rb_g of every group of the share, from shared memory;
+//   probe   each lane set races its lowest-bound group exactly (the drafter
+//           vectors are the only logits read from memory besides the
+//           target row); K1, the least of these keys over the cluster, is
+//           exchanged through distributed shared memory;
+//   race    every group whose bound does not put it above K1 (U_g f > K1 Rb_g
+//           fails, f = kRaceFilter) is raced exactly, with the arithmetic and
+//           summation order of the race over every group;
+//   level 2 the cluster's least (key, group), lowest group on ties, gets the
+//           entry race.
+// A group left out has a key above K1 by more than the filter's margin (1e-5
+// relative, far above the rounding of E, of the sum and of the quotient), so
+// it can neither win nor tie: the token is the one the race over every group
+// draws.  The drafter row and the exponentials are touched for a few groups
+// per row instead of all of them.
+#ifndef CMSD_CLU_CTAS
+#define CMSD_CLU_CTAS 4
+#endif
+constexpr int kCluCtas = CMSD_CLU_CTAS;                  // CTAs per row (one cluster)
+constexpr int kCluThreads = 512;
+constexpr int kCluWarps = kCluThreads / 32;
+constexpr int kCluCands = 1024;                          // candidate list; past it the share is raced whole
+constexpr size_t kCluSmemMax = 200 * 1024;               // larger shares take the race over every group
+constexpr float kGroupBoundScale = 32.0f + 1.0f / 2048.0f;   // kGroup (1 + 2^-16)
+constexpr float kGroupBoundFloor = 0x1p-100f;
+static_assert(kGroup == 32, "the bound's factor is kGroup (1 + 2^-16)");
+
+// Groups per CTA: a multiple of four, so that a share starts on a block of
+// four group uniforms.
+__host__ __device__ inline int clu_share(int ng) {
+  const int s = (ng + kCluCtas - 1) / kCluCtas;
+  return (s + 3) & ~3;
+}
+// Dynamic shared memory of one CTA: the staged target share, the share's
+// uniforms and bounds, the candidate list.
+template <typename T>
+__host__ __device__ inline size_t clu_smem_bytes(int V) {
+  const size_t ngs = (size_t)clu_share((V + kGroup - 1) / kGroup);
+  return ngs * kGroup * sizeof(T) + ngs * 2 * sizeof(float) + (size_t)kCluCands * sizeof(int);
+}
+
+__device__ __forceinline__ float expo_u(float u) { return -log1pf(-u); }   // expo() of the same word
+
+// The largest logit of a 16-byte vector.
+__device__ __forceinline__ float vec_max(uint4 q, const uint16_t*) {
+  const uint32_t m = bmax2(bmax2(q.x, q.y), bmax2(q.z, q.w));
+  return fmaxf(bf_lo(m), bf_hi(m));
+}
+__device__ __forceinline__ float vec_max(uint4 q, const float*) {
+  return fmaxf(fmaxf(__uint_as_float(q.x), __uint_as_float(q.y)), fmaxf(__uint_as_float(q.z), __uint_as_float(q.w)));
+}
+
+// The staged share keeps group g's vectors in 16-byte slots g LPG .. g LPG +
+// LPG - 1, vector k in slot g LPG + ((k + rot(g)) mod LPG), rot(g) = g LPG / 8:
+// a thread that reads a whole group (one vector per load) and its neighbours
+// reading theirs then touch eight different 16-byte bank slots per quarter
+// warp.
+template <int LPG>
+__device__ __forceinline__ int clu_slot(int g, int k) {
+  return g * LPG + ((k + ((g * LPG) >> 3)) & (LPG - 1));
+}
+
+// The largest logit of staged group g.
+__device__ __forceinline__ float group_max(const unsigned char* stage, int g, const uint16_t*) {
+  const uint4* q = reinterpret_cast<const uint4*>(stage);
+  const uint4 a = q[clu_slot<4>(g, 0)], b = q[clu_slot<4>(g, 1)], c = q[clu_slot<4>(g, 2)], d = q[clu_slot<4>(g, 3)];
+  const uint32_t x = bmax2(bmax2(a.x, b.x), bmax2(c.x, d.x));
+  const uint32_t y = bmax2(bmax2(a.y, b.y), bmax2(c.y, d.y));
+  const uint32_t z = bmax2(bmax2(a.z, b.z), bmax2(c.z, d.z));
+  const uint32_t w = bmax2(bmax2(a.w, b.w), bmax2(c.w, d.w));
+  const uint32_t m = bmax2(bmax2(x, y), bmax2(z, w));
+  return fmaxf(bf_lo(m), bf_hi(m));
+}
+__device__ __forceinline__ float group_max(const unsigned char* stage, int g, const float*) {
+  const uint4* q = reinterpret_cast<const uint4*>(stage);
+  float m = -pos_inf();
+#pragma unroll
+  for (int k = 0; k < 8; ++k) m = fmaxf(m, vec_max(q[clu_slot<8>(g, k)], (const float*)nullptr));
+  return m;
+}
+
+// Rb_g from the group's largest target logit.
+__device__ __forceinline__ float group_bound(float m, const RowStat& st) {
+  const float pm = __fmul_rn(ex2(__fmaf_rn(m, kLog2e, -st.MLt)), st.invSt);
+  return __fmaf_rn(pm, kGroupBoundScale, kGroupBoundFloor);
+}
+
+// (key, group) order: the least key, the lowest group on ties.
+__device__ __forceinline__ void key_min(float& k, int& g, float k2, int g2) {
+  if (k2 < k || (k2 == k && g2 < g)) {
+    k = k2;
+    g = g2;
+  }
+}
+// The CTA's least (key, group) in every thread, keys >= 0 or +inf and groups
+// >= 0 or kIntMax: the pair ordered as one 64-bit integer (key bits, group),
+// a redux.sync minimum per warp and one shared-memory atomicMin per warp.
+// *s_best holds ~0 on entry (reset behind a barrier) and is read by every
+// thread before the function returns.
+__device__ __forceinline__ void key_min_cta(float& k, int& g, unsigned long long* s_best) {
+  const uint32_t kb = __reduce_min_sync(kFull, __float_as_uint(k));
+  const uint32_t gb = __reduce_min_sync(kFull, __float_as_uint(k) == kb ? (uint32_t)g : 0xFFFFFFFFu);
+  if ((threadIdx.x & 31) == 0) atomicMin(s_best, ((unsigned long long)kb << 32) | gb);
+  __syncthreads();
+  const unsigned long long v = *s_best;
+  k = __uint_as_float((uint32_t)(v >> 32));
+  g = (int)(uint32_t)v;
+}
+
+// The exact key of a group from its vectors (vector `sub` in lane `sub` of
+// the lane set; target qt, drafter qd): the sum in the order of the race over
+// every group.  +inf when the residual mass is zero or `ok` is false.
+template <typename T>
+__device__ __forceinline__ float group_key(uint4 qt, uint4 qd, const RowStat& st, float u, bool ok) {
+  constexpr int LPG = kGroup / Elem<T>::kVec;
+  float acc = resid_vec<T>(qt, qd, st);
+#pragma unroll
+  for (int o = 1; o < LPG; o <<= 1) acc += __shfl_xor_sync(kFull, acc, o);
+  return (ok && acc > 0.f) ? expo_u(u) / acc : pos_inf();
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kCluThreads, 2) resample_bound_kernel(const StreamArgs a) {
+  constexpr int VEC = Elem<T>::kVec;
+  constexpr int LPG = kGroup / VEC;      // lanes per group
+  constexpr int GPI = 32 / LPG;          // lane sets per warp
+  constexpr int SETS = kCluWarps * GPI;  // lane sets per CTA
+  extern __shared__ __align__(16) unsigned char clu_smem[];
+  __shared__ unsigned long long s_best[2];   // key_min_cta of the probes, of the race
+  __shared__ int s_n, s_hold;
+  __shared__ int s_probe[SETS];          // the group each lane set probed (a group of one of its threads)
+  __shared__ uint4 s_qd[SETS * LPG];     // drafter vectors of each lane set's best group
+  __shared__ float s_k1[kCluCtas];       // each CTA's least probe key, written by that CTA into every CTA
+  __shared__ float s_rk[kCluCtas];       // rank 0: each CTA's (key, group, token)
+  __shared__ int s_rg[kCluCtas];
+  __shared__ int s_rt[kCluCtas];
+  cg::cluster_group cl = cg::this_cluster();
+  const int cr = (int)cl.block_rank();
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const int sub = lane % LPG;
+  const int set = warp * GPI + lane / LPG;
+  const int ng = (a.V + kGroup - 1) / kGroup;
+  const int ngs = clu_share(ng);
+  unsigned char* stage = clu_smem;
+  float* s_u = reinterpret_cast<float*>(clu_smem + (size_t)ngs * kGroup * sizeof(T));
+  float* s_rb = s_u + ngs;
+  int* s_list = reinterpret_cast<int*>(s_rb + ngs);
+  const int gs = cr * ngs;                                   // the share: groups [gs, gs + nloc)
+  const int nloc = max(0, min(ng, gs + ngs) - gs);
+  const uint32_t k0 = seed_lo(a.seed), k1 = seed_hi(a.seed);
+  const uint32_t cw_grp = iter_word(a.iteration, kPurposeGroup);
+  const uint32_t cw_ent = iter_word(a.iteration, kPurposeResidual);
+  const int ncl = (int)gridDim.x / kCluCtas;
+  const int rr0 = (int)blockIdx.x / kCluCtas;
+  // everything below reads what the streaming kernel wrote; the queue length
+  // and the cluster's first record are read together
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const Workspace& W = a.ws;
+  int R = __ldcg(W.rec_count);
+  int4 rec = rr0 < a.B ? __ldcg(W.rec + rr0) : make_int4(0, 0, kSeqNone, 0);
+  R = R < 0 ? 0 : (R > a.B ? a.B : R);
+  // Two cluster barriers per row: after the probes (K1) and after the
+  // results.  A slot written before one barrier is read only between it and
+  // the next, so no row overwrites what the previous row still reads.
+  for (int rr = rr0; rr < R; rr += ncl) {                    // the same rows for the whole cluster
+    if (rr != rr0) rec = __ldcg(W.rec + rr);
+    if (rec.z != kSeqResidual) continue;   // only residual rows are queued without the bonus row
+    const int b = rec.x, pos = rec.y;
+    const int r = b * a.K + pos;
+    const T* tp = (const T*)a.target + (size_t)r * (size_t)a.V;     // no bonus row: Kt == K
+    const T* dp = (const T*)a.draft + (size_t)r * (size_t)a.V;
+    const bool vec_ok = ((((uintptr_t)tp) | ((uintptr_t)dp)) & 15) == 0;
+    if (threadIdx.x == 0) s_best[0] = s_best[1] = ~0ull;   // the last row read them before its barriers
+    // stage: the share of the target row (-inf past the row end), while the
+    // share's uniforms are drawn and the row statistics load
+    const int v0 = gs * kGroup;
+    for (int j = threadIdx.x; j < nloc * LPG; j += kCluThreads) {
+      const int v = v0 + j * VEC;
+      const int sl = clu_slot<LPG>(j / LPG, j % LPG);
+      if (vec_ok && v + VEC <= a.V) cp_async16(smem_u32(stage) + 16u * (uint32_t)sl, tp + v);
+      else *reinterpret_cast<uint4*>(stage + 16 * sl) = load_logits<T>(tp, v, a.V, false);
+    }
+    cp_async_commit();
+    const float2 ts = __ldcg(W.row_tstat + r), ds = __ldcg(W.row_dstat + r);
+    for (int q = threadIdx.x; q < (nloc + 3) / 4; q += kCluThreads) {
+      const U4 wd = philox4x32_10(U4{(uint32_t)(gs / 4 + q), (uint32_t)b, (uint32_t)pos, cw_grp}, k0, k1);
+      s_u[4 * q + 0] = word_to_unit(wd.x);
+      s_u[4 * q + 1] = word_to_unit(wd.y);
+      s_u[4 * q + 2] = word_to_unit(wd.z);
+      s_u[4 * q + 3] = word_to_unit(wd.w);
+    }
+    const RowStat st{ts.x, 1.0f / ts.y, ds.x, -1.0f / ds.y};
+    cp_async_wait<0>();
+    __syncthreads();
+    // bound: m_g and Rb_g, one thread per group; each thread keeps its
+    // lowest U_g / Rb_g (compared as U_a Rb_b < U_b Rb_a), then each lane set
+    // the lowest of its LPG threads'
+    float bu = 0.f, brb = 1.f;
+    int lg = -1;
+    for (int gl = threadIdx.x; gl < nloc; gl += kCluThreads) {
+      const float rb = group_bound(group_max(stage, gl, (const T*)nullptr), st);
+      s_rb[gl] = rb;
+      const float u = s_u[gl];
+      if (lg < 0 || u * brb < bu * rb) {
+        bu = u;
+        brb = rb;
+        lg = gl;
+      }
+    }
+#pragma unroll
+    for (int o = 1; o < LPG; o <<= 1) {
+      const float u2 = __shfl_xor_sync(kFull, bu, o), rb2 = __shfl_xor_sync(kFull, brb, o);
+      const int g2 = __shfl_xor_sync(kFull, lg, o);
+      if (g2 >= 0 && (lg < 0 || u2 * brb < bu * rb2 || (u2 * brb == bu * rb2 && g2 < lg))) {
+        bu = u2;
+        brb = rb2;
+        lg = g2;
+      }
+    }
+    // probe: the lane set's lowest-bound group, exactly
+    float sk;                              // the lane set's best (key, group), its drafter vectors in s_qd
+    int sg;
+    {
+      uint4 qt = neg_inf_vec<T>(), qd = neg_inf_vec<T>();
+      if (lg >= 0) {
+        qt = *reinterpret_cast<const uint4*>(stage + 16 * clu_slot<LPG>(lg, sub));
+        qd = load_logits<T>(dp, (gs + lg) * kGroup + sub * VEC, a.V, vec_ok);
+      }
+      sk = group_key<T>(qt, qd, st, lg >= 0 ? s_u[lg] : 0.f, lg >= 0);
+      sg = sk != pos_inf() ? gs + lg : kIntMax;
+      s_qd[set * LPG + sub] = qd;
+      if (sub == 0) s_probe[set] = lg;
+    }
+    float K1 = sk;
+    int g1 = sg;
+    key_min_cta(K1, g1, &s_best[0]);
+    // K1: the least probe key of the cluster, an upper bound on the winner's key
+    if (threadIdx.x < kCluCtas) *cl.map_shared_rank(&s_k1[cr], (int)threadIdx.x) = K1;
+    if (threadIdx.x == 0) s_n = 0;
+    cl.sync();
+#pragma unroll
+    for (int c = 0; c < kCluCtas; ++c) K1 = fminf(K1, s_k1[c]);
+    // race: the groups of the share that the bound leaves at or below K1 and
+    // that no lane set has probed (s_rb is complete: the barriers above)
+    for (int gl = threadIdx.x; gl < nloc; gl += kCluThreads) {
+      if (!(s_u[gl] * kRaceFilter > K1 * s_rb[gl]) && s_probe[(gl % kCluThreads) / LPG] != gl) {
+        const int i = atomicAdd(&s_n, 1);
+        if (i < kCluCands) s_list[i] = gl;
+      }
+    }
+    __syncthreads();
+    const int nc = s_n;
+    const bool whole = nc > kCluCands;
+    const int items = whole ? nloc : nc;
+    for (int i0 = 0; i0 < items; i0 += SETS) {               // warp-uniform trip count
+      const int i = i0 + set;
+      const int gl = i < items ? (whole ? i : s_list[i]) : -1;
+      uint4 qt = neg_inf_vec<T>(), qd = neg_inf_vec<T>();
+      if (gl >= 0) {
+        qt = *reinterpret_cast<const uint4*>(stage + 16 * clu_slot<LPG>(gl, sub));
+        qd = load_logits<T>(dp, (gs + gl) * kGroup + sub * VEC, a.V, vec_ok);
+      }
+      const float key = group_key<T>(qt, qd, st, gl >= 0 ? s_u[gl] : 0.f, gl >= 0);
+      if (key != pos_inf() && (key < sk || (key == sk && gs + gl < sg))) {   // the whole lane set agrees
+        sk = key;
+        sg = gs + gl;
+        s_qd[set * LPG + sub] = qd;
+      }
+    }
+    // the CTA's least (key, group), the lane set holding it, and its level-2
+    // winner, pushed to rank 0 of the cluster
+    float ck = sk;
+    int cgrp = sg;
+    if (threadIdx.x == 0) s_hold = 0;
+    key_min_cta(ck, cgrp, &s_best[1]);
+    if (sub == 0 && cgrp != kIntMax && sk == ck && sg == cgrp) s_hold = set;   // holders share one vector set
+    __syncthreads();
+    if (warp == 0) {
+      int tok = -1;
+      if (cgrp != kIntMax) {
+        const int h = s_hold;
+        const uint4 qt = *reinterpret_cast<const uint4*>(stage + 16 * clu_slot<LPG>(cgrp - gs, sub));
+        const uint4 qd = s_qd[h * LPG + sub];
+        tok = race_group_entries<T>(qt, qd, cgrp, 0, lane, st, (uint32_t)b, (uint32_t)pos, cw_ent, k0, k1);
+      }
+      if (lane == 0) {
+        *cl.map_shared_rank(&s_rk[cr], 0) = ck;
+        *cl.map_shared_rank(&s_rg[cr], 0) = cgrp;
+        *cl.map_shared_rank(&s_rt[cr], 0) = tok;
+      }
+    }
+    cl.sync();                             // every CTA's result is in rank 0
+    if (cr == 0 && threadIdx.x == 0) {
+      float k = pos_inf();
+      int g = kIntMax, tok = -1;
+#pragma unroll 1
+      for (int c = 0; c < kCluCtas; ++c) {
+        const float kc = s_rk[c];
+        const int gc = s_rg[c];
+        if (kc < k || (kc == k && gc < g)) {
+          k = kc;
+          g = gc;
+          tok = s_rt[c];
+        }
+      }
+      if (g == kIntMax || tok < 0) tok = __ldcg(W.row_targmax + r);   // empty residual: the argmax
+      a.out_tokens[(size_t)b * a.Ko + pos] = tok;
+    }
+  }
+  // the last CTA to finish clears the queue for the next call
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int done = atom_add_acq_rel(W.res_cta_done, 1);
+    if (done == (int)gridDim.x - 1) {
+      *W.rec_count = 0;
+      *W.res_cta_done = 0;
+      __threadfence();
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // the kernel
 // ---------------------------------------------------------------------------
 
@@ -1722,6 +2062,37 @@ cudaError_t launch_resample_one(const StreamArgs& a, int grid, cudaStream_t s) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, resample_kernel<T, SAMPLED>, a);
+}
+
+// The residual draw by group bounds: `clusters` clusters of kCluCtas CTAs,
+// launched the same way (the row loop covers any number of queued rows).
+template <typename T>
+cudaError_t launch_resample_bound_t(const StreamArgs& a, int clusters, cudaStream_t s) {
+  static unsigned long long done = 0ull;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (!(__atomic_load_n(&done, __ATOMIC_ACQUIRE) & bit)) {
+    e = cudaFuncSetAttribute(resample_bound_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kCluSmemMax);
+    if (e != cudaSuccess) return e;
+    __atomic_fetch_or(&done, bit, __ATOMIC_ACQ_REL);
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(clusters * kCluCtas));
+  cfg.blockDim = dim3(kCluThreads);
+  cfg.dynamicSmemBytes = clu_smem_bytes<T>(a.V);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = kCluCtas;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, resample_bound_kernel<T>, a);
 }
 
 template <typename T>
