@@ -7,8 +7,10 @@ per-row permutation + 0.5 N(0,1); target = drafter + N(0,1); drafted tokens
 sampled from the drafter), SAMPLED rule (Philox acceptance + residual draw).
 
 A step is one call of cmsd_confidence_verify over one batch: the streaming
-kernel (every drafter and target logit read once) plus the resample kernel
-over the rejected row pair of each sequence.  Two distinct input sets
+kernel (every drafter and target logit read once) plus the residual draw at
+each sequence's rejected position (a cluster of CTAs per row: the target row
+again, and the drafter logits of the few groups the bound keeps).  Two
+distinct input sets
 (2 x 263 MB, each larger than the 129 MB L2) alternate between steps.
 
 Besides the headline, one JSON line carries (rank 0, one GPU): the other
@@ -89,6 +91,7 @@ def ncu_traffic(workload, rule):
         recs = recs if isinstance(recs, list) else [recs]
         for d in recs:
             if d.get("workload") == workload and d.get("rule") == rule and \
+                    d.get("kernel", "").startswith("stream_kernel") and \
                     d.get("sources_sha256_16") == kernel_sources_sha():
                 return d.get("bytes_per_launch")
     except Exception:
@@ -392,7 +395,7 @@ def bench_workload(cmsd, torch, dev, name, rule, steps, peak, nsets=1, graph_lat
            "kernel_ms": km, "resample_ms": statistics.median(r_ms) if rule == "sampled" else 0.0,
            "algorithmic_bytes": alg, "kernel_gbs": alg / (km * 1e-3) / 1e9,
            "kernel_frac": alg / (km * 1e-3) / 1e9 / peak,
-           "step_gbs": (alg + rejected * 2 * V * es) / (total / steps * 1e-3) / 1e9,
+           "step_gbs": (alg + rejected * V * es) / (total / steps * 1e-3) / 1e9,   # + the rejected target rows
            "l2": "inputs larger than L2" if alg > 129e6 else "L2-resident (inputs smaller than L2)",
            "traffic": ncu_traffic(name, rule), "parity": parity_record(name, rule)}
     res["step_frac"] = res["step_gbs"] / peak
@@ -723,7 +726,9 @@ def run_ours(args):
     k_med = statistics.median(k_ms)
     achieved = alg_bytes / (k_med * 1e-3) / 1e9
     step_stats = stats_ms(per_step)
-    resample_bytes = rejected * 2 * V * 2
+    # the residual draw reads each rejected position's target row again (the
+    # drafter groups it races are a few KB)
+    resample_bytes = rejected * V * 2
     step_gbs = (alg_bytes + resample_bytes) / (ms_step * 1e-3) / 1e9
 
     if rank != 0:
@@ -782,7 +787,8 @@ def run_ours(args):
         "step_roofline": {"achieved": step_gbs, "frac": step_gbs / peak, "unit": "GB/s",
                           "bytes_per_step": alg_bytes + resample_bytes,
                           "resample_bytes_per_step": resample_bytes,
-                          "note": "every logit once plus the rejected row pairs again, over the median step"},
+                          "note": "every logit once plus the rejected positions' target rows again, over the "
+                                  "median step"},
         "resample_ms": statistics.median(r_ms) if sampled else 0.0,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,

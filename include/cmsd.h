@@ -211,8 +211,9 @@ int cmsd_verify(const void* draft_logits, const void* target_logits,
 
 /*
  * The fused pass: cmsd_confidence and cmsd_verify in one streaming read of
- * both logit tensors (plus a second pass over the rejected row pair, or the
- * bonus row, of each sequence that needs one).  Same arguments
+ * both logit tensors (plus a second pass over the rejected position of each
+ * sequence that needs one -- its target row and the drafter logits of the
+ * groups the draw races -- or over the bonus row).  Same arguments
  * and outputs as the two calls above; n_accept and out_tokens are required,
  * the rest may be NULL.
  */

@@ -1613,8 +1613,14 @@ __global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_ker
 #ifndef CMSD_CLU_CTAS
 #define CMSD_CLU_CTAS 4
 #endif
+#ifndef CMSD_CLU_THREADS
+#define CMSD_CLU_THREADS 512
+#endif
+#ifndef CMSD_CLU_MIN_BLOCKS
+#define CMSD_CLU_MIN_BLOCKS 2
+#endif
 constexpr int kCluCtas = CMSD_CLU_CTAS;                  // CTAs per row (one cluster)
-constexpr int kCluThreads = 512;
+constexpr int kCluThreads = CMSD_CLU_THREADS;
 constexpr int kCluWarps = kCluThreads / 32;
 constexpr int kCluCands = 1024;                          // candidate list; past it the share is raced whole
 constexpr size_t kCluSmemMax = 200 * 1024;               // larger shares take the race over every group
@@ -1717,7 +1723,7 @@ __device__ __forceinline__ float group_key(uint4 qt, uint4 qd, const RowStat& st
 }
 
 template <typename T>
-__global__ void __launch_bounds__(kCluThreads, 2) resample_bound_kernel(const StreamArgs a) {
+__global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bound_kernel(const StreamArgs a) {
   constexpr int VEC = Elem<T>::kVec;
   constexpr int LPG = kGroup / VEC;      // lanes per group
   constexpr int GPI = 32 / LPG;          // lane sets per warp
@@ -1795,6 +1801,7 @@ __global__ void __launch_bounds__(kCluThreads, 2) resample_bound_kernel(const St
     // the lowest of its LPG threads'
     float bu = 0.f, brb = 1.f;
     int lg = -1;
+#pragma unroll 2
     for (int gl = threadIdx.x; gl < nloc; gl += kCluThreads) {
       const float rb = group_bound(group_max(stage, gl, (const T*)nullptr), st);
       s_rb[gl] = rb;
