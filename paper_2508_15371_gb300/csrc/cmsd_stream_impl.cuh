@@ -41,9 +41,13 @@
 // from the residual max(0, p - q), and with the bonus row the verifier's extra
 // row gives a token when every draft was accepted; both need one more pass
 // over one row of the sequence after its epilogue.  The epilogue queues a
-// record for each sequence that needs one; the resample kernel, launched as a
-// programmatic dependent of this one, splits the queued rows' groups evenly
-// over its warps.  Every logit of the pass proper is read once.
+// record for each sequence that needs one; a second kernel, launched as a
+// programmatic dependent of this one, drains the queue: under the sampled rule
+// without the bonus row, resample_bound_kernel (a cluster of CTAs per row that
+// bounds each group's residual mass by its largest target logit and races
+// only the groups the bound leaves in play); otherwise resample_kernel (the
+// queued rows' groups split evenly over its warps, every group raced).  Every
+// logit of the pass proper is read once.
 //
 // -inf logits (masked vocabulary) are clamped to -2^100 before the drafter
 // arithmetic so that e^(z-m) * (z-m) is 0, not NaN.
