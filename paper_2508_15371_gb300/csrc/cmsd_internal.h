@@ -121,7 +121,8 @@ cudaError_t launch_resample_f32(bool sampled, const StreamArgs& a, int grid, cud
 cudaError_t launch_resample_bf16(bool sampled, const StreamArgs& a, int grid, cudaStream_t s);
 // The residual draw by group bounds (sampled rule, no bonus row): clusters
 // of CTAs, one queued row per cluster at a time; resample_bound_fits says
-// whether a row's share fits its shared memory (else resample_kernel).
+// whether a row's share fits its shared memory and such a cluster can be
+// resident on the current device (else resample_kernel draws the residual).
 cudaError_t launch_resample_bound_f32(const StreamArgs& a, int clusters, cudaStream_t s);
 cudaError_t launch_resample_bound_bf16(const StreamArgs& a, int clusters, cudaStream_t s);
 bool resample_bound_fits(int dtype, int V);

@@ -20,6 +20,8 @@ cudaError_t launch_resample_bound_bf16(const StreamArgs& a, int clusters, cudaSt
   return launch_resample_bound_t<uint16_t>(a, clusters, s);
 }
 
+bool resample_bound_fits_bf16(int V) { return resample_bound_fits_t<uint16_t>(V); }
+
 cudaError_t occupancy_resample_bf16(bool sampled, int* nb) { return occupancy_resample_t<uint16_t>(sampled, nb); }
 
 }  // namespace cmsd

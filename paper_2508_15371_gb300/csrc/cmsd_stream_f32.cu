@@ -15,8 +15,9 @@ cudaError_t launch_resample_bound_f32(const StreamArgs& a, int clusters, cudaStr
   return launch_resample_bound_t<float>(a, clusters, s);
 }
 
+bool resample_bound_fits_bf16(int V);
 bool resample_bound_fits(int dtype, int V) {
-  return (dtype == 0 ? clu_smem_bytes<float>(V) : clu_smem_bytes<uint16_t>(V)) <= kCluSmemMax;
+  return dtype == 0 ? resample_bound_fits_t<float>(V) : resample_bound_fits_bf16(V);
 }
 
 cudaError_t occupancy_resample(int dtype, bool sampled, int* nb) {

@@ -53,6 +53,9 @@
 // arithmetic so that e^(z-m) * (z-m) is 0, not NaN.
 #pragma once
 #include <cooperative_groups.h>
+#include <map>
+#include <mutex>
+#include <utility>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -1916,11 +1919,13 @@ __global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bou
       a.out_tokens[(size_t)b * a.Ko + pos] = tok;
     }
   }
-  // the last CTA to finish clears the queue for the next call
-  __syncthreads();
-  if (threadIdx.x == 0) {
+  // The last cluster to finish clears the queue for the next call.  Rank 0
+  // counts for its cluster: with rows, after the cluster's last barrier, when
+  // every CTA of it has read the queue length; without, a CTA that reads the
+  // cleared length still finds no row of its own.
+  if (cr == 0 && threadIdx.x == 0) {
     const int done = atom_add_acq_rel(W.res_cta_done, 1);
-    if (done == (int)gridDim.x - 1) {
+    if (done == ncl - 1) {
       *W.rec_count = 0;
       *W.res_cta_done = 0;
       __threadfence();
@@ -2104,6 +2109,44 @@ cudaError_t launch_resample_bound_t(const StreamArgs& a, int clusters, cudaStrea
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, resample_bound_kernel<T>, a);
+}
+
+// Whether the residual draw by group bounds takes rows of V entries on the
+// current device: the share fits kCluSmemMax, and a cluster of kCluCtas CTAs
+// with that much shared memory can be resident (answer cached per device and
+// size).  Otherwise resample_kernel draws the residual.
+template <typename T>
+bool resample_bound_fits_t(int V) {
+  const size_t smem = clu_smem_bytes<T>(V);
+  if (smem > kCluSmemMax) return false;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  static std::mutex mu;
+  static std::map<std::pair<int, size_t>, bool> cache;
+  std::lock_guard<std::mutex> lk(mu);
+  const auto key = std::make_pair(dev, smem);
+  const auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  bool ok = false;
+  if (cudaFuncSetAttribute(resample_bound_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)kCluSmemMax) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kCluCtas);
+    cfg.blockDim = dim3(kCluThreads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = kCluCtas;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    ok = cudaOccupancyMaxActiveClusters(&n, resample_bound_kernel<T>, &cfg) == cudaSuccess && n > 0;
+  }
+  if (!ok) (void)cudaGetLastError();   // a refused query leaves no error behind for the caller
+  cache.emplace(key, ok);
+  return ok;
 }
 
 template <typename T>
