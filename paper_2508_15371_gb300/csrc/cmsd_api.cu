@@ -260,6 +260,7 @@ int launch(int dtype, int mode, bool sampled, StreamArgs& a, void* ws, size_t ws
     nclu = a.B < 2 * sms ? a.B : 2 * sms;
   }
   a.nwarps = grid * kStreamWarps;
+  a.rec_by_seq = bound ? 1 : 0;
   prof_record(0, s);
   cudaError_t e = dtype == CMSD_F32 ? launch_stream_f32(mode, sampled, second, a, grid, smem, s)
                                     : launch_stream_bf16(mode, sampled, second, a, grid, smem, s);

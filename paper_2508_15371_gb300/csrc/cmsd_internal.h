@@ -109,6 +109,8 @@ struct StreamArgs {
   unsigned char* accept;
   Workspace ws;
   int nwarps;             // warps launched
+  int rec_by_seq;         // 1: second-pass records at each sequence's own slot rec[b], every sequence
+                          // writing one (the bounded residual draw); 0: a compacted queue (rec_count)
 };
 
 // Kernel launchers (one translation unit per dtype).  `second`: this call

@@ -603,8 +603,14 @@ __device__ __forceinline__ int next_k(const StreamArgs& a, unsigned long long cs
   return k < a.k_min ? a.k_min : k;
 }
 
-// Queue the sequence's second-pass record, if it needs one.
+// Queue the sequence's second-pass record, if it needs one; or, for the
+// bounded residual draw, write it (kSeqNone included) at the sequence's own
+// slot, with no atomic round trip at the end of the epilogue.
 __device__ __forceinline__ void publish(const StreamArgs& a, int b, int kind, int pos) {
+  if (a.rec_by_seq) {
+    a.ws.rec[b] = make_int4(b, pos, kind, 0);
+    return;
+  }
   if (kind == kSeqNone) return;
   const int slot = atomicAdd(a.ws.rec_count, 1);
   if (slot < a.B) a.ws.rec[slot] = make_int4(b, pos, kind, 0);
@@ -1598,8 +1604,9 @@ __global__ void __launch_bounds__(kResThreads, CMSD_RES_MIN_BLOCKS) resample_ker
 //   R_g <= Rb_g = kGroup p(m_g) (1 + 2^-16) + 2^-100
 // (the factor covers the rounding of the 32-term sum and of ex2, the floor
 // entries whose p underflows), and its key E_g / R_g >= U_g / Rb_g because
-// E = -log(1 - U) >= U.  A cluster of kCluCtas CTAs takes one queued row, a
-// share of its groups each:
+// E = -log(1 - U) >= U.  A cluster of kCluCtas CTAs takes one sequence's
+// rejected row (its record at the sequence's own slot), a share of its groups
+// each:
 //   stage   the share of the target row is copied to shared memory (cp.async)
 //           while the share's uniforms are drawn;
 //   bound   m_g and Rb_g of every group of the share, from shared memory;
@@ -1762,20 +1769,16 @@ __global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bou
   const uint32_t cw_grp = iter_word(a.iteration, kPurposeGroup);
   const uint32_t cw_ent = iter_word(a.iteration, kPurposeResidual);
   const int ncl = (int)gridDim.x / kCluCtas;
-  const int rr0 = (int)blockIdx.x / kCluCtas;
-  // everything below reads what the streaming kernel wrote; the queue length
-  // and the cluster's first record are read together
+  // everything below reads what the streaming kernel wrote: every sequence's
+  // record at its own slot (rec_by_seq)
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const Workspace& W = a.ws;
-  int R = __ldcg(W.rec_count);
-  int4 rec = rr0 < a.B ? __ldcg(W.rec + rr0) : make_int4(0, 0, kSeqNone, 0);
-  R = R < 0 ? 0 : (R > a.B ? a.B : R);
   // Two cluster barriers per row: after the probes (K1) and after the
   // results.  A slot written before one barrier is read only between it and
   // the next, so no row overwrites what the previous row still reads.
-  for (int rr = rr0; rr < R; rr += ncl) {                    // the same rows for the whole cluster
-    if (rr != rr0) rec = __ldcg(W.rec + rr);
-    if (rec.z != kSeqResidual) continue;   // only residual rows are queued without the bonus row
+  for (int rr = (int)blockIdx.x / kCluCtas; rr < a.B; rr += ncl) {   // sequence rr, the same for the cluster
+    const int4 rec = __ldcg(W.rec + rr);
+    if (rec.z != kSeqResidual) continue;   // no residual draw for this sequence in this call
     const int b = rec.x, pos = rec.y;
     const int r = b * a.K + pos;
     const T* tp = (const T*)a.target + (size_t)r * (size_t)a.V;     // no bonus row: Kt == K
@@ -1919,18 +1922,7 @@ __global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bou
       a.out_tokens[(size_t)b * a.Ko + pos] = tok;
     }
   }
-  // The last cluster to finish clears the queue for the next call.  Rank 0
-  // counts for its cluster: with rows, after the cluster's last barrier, when
-  // every CTA of it has read the queue length; without, a CTA that reads the
-  // cleared length still finds no row of its own.
-  if (cr == 0 && threadIdx.x == 0) {
-    const int done = atom_add_acq_rel(W.res_cta_done, 1);
-    if (done == ncl - 1) {
-      *W.rec_count = 0;
-      *W.res_cta_done = 0;
-      __threadfence();
-    }
-  }
+  // (the per-sequence slots need no clearing: every call writes all of them)
 }
 
 // ---------------------------------------------------------------------------
