@@ -875,6 +875,13 @@ __device__ void seg_finish(const StreamArgs& a, SegState& ss, int ar, int r, int
   // the loads overlap the shuffles: there the kernel's tail is this latency,
   // and the early requests measured 3 us faster than the late ones.
   const float me = HAS_D ? d_mexp(ss.d) : 0.f;
+  // Under the sampled rule the exact indices feed only the drafter's argmax
+  // output and resample_kernel's empty-residual fallback (the bounded draw
+  // finds that argmax itself): without them a lane's vector start stands in
+  // (distinct per lane and ordered like the index, so the merges still tell
+  // the maximum's lane from a duplicate of its value) and nothing is re-read.
+  const bool want_didx = !SAMPLED || a.argmax != nullptr;
+  const bool want_tidx = !SAMPLED || !a.rec_by_seq;
   uint4 dq = make_uint4(0, 0, 0, 0), tq = make_uint4(0, 0, 0, 0);
   if (!SAMPLED) {
     if (HAS_D && ss.d.posw > 1) dq = __ldcg(reinterpret_cast<const uint4*>(dp + ss.d.pos));
@@ -884,8 +891,8 @@ __device__ void seg_finish(const StreamArgs& a, SegState& ss, int ar, int r, int
   const float Mt = HAS_T ? warp_max(ss.t.M) : 0.f;
   const bool dhit = HAS_D && me == Md && ss.d.posw, thit = HAS_T && ss.t.M == Mt && ss.t.posw;
   if (SAMPLED) {
-    if (dhit && ss.d.posw > 1) dq = __ldcg(reinterpret_cast<const uint4*>(dp + ss.d.pos));
-    if (thit && ss.t.posw > 1) tq = __ldcg(reinterpret_cast<const uint4*>(tp + ss.t.pos));
+    if (want_didx && dhit && ss.d.posw > 1) dq = __ldcg(reinterpret_cast<const uint4*>(dp + ss.d.pos));
+    if (want_tidx && thit && ss.t.posw > 1) tq = __ldcg(reinterpret_cast<const uint4*>(tp + ss.t.pos));
   }
   DRed dr = dred_empty();
   TRed tr = tred_empty();
@@ -901,13 +908,13 @@ __device__ void seg_finish(const StreamArgs& a, SegState& ss, int ar, int r, int
     float s, t2;
     d_final(d, s, t2);
     int idx = kIntMax;
-    if (dhit) idx = d.posw > 1 ? d.pos + first_in_vec<T>(dq, me, true) : d.pos;
+    if (dhit) idx = (want_didx && d.posw > 1) ? d.pos + first_in_vec<T>(dq, me, true) : d.pos;
     dr = reduce_d(DRed{me, s, t2, top2, idx});
   }
   if (HAS_T) {
     const TLane& t = ss.t;
     int idx = kIntMax;
-    if (thit) idx = t.posw > 1 ? t.pos + first_in_vec<T>(tq, t.M, false) : t.pos;
+    if (thit) idx = (want_tidx && t.posw > 1) ? t.pos + first_in_vec<T>(tq, t.M, false) : t.pos;
     tr = reduce_t(TRed{t.M, SAMPLED ? t_final(t) : 0.f, idx, t.cnt});
   }
   // lane 0 stores the partial and counts it with a release; the warp that
@@ -1736,6 +1743,36 @@ __device__ __forceinline__ float group_key(uint4 qt, uint4 qd, const RowStat& st
   return (ok && acc > 0.f) ? expo_u(u) / acc : pos_inf();
 }
 
+// The verifier row's argmax (the lowest index of its largest logit), by the
+// whole CTA from global memory: the token of a row whose residual is empty.
+// *s_am holds 0 on entry (reset behind a barrier).
+template <typename T>
+__device__ int row_argmax_cta(const T* tp, int V, bool vec_ok, unsigned long long* s_am) {
+  constexpr int VEC = Elem<T>::kVec;
+  float bm = -pos_inf();
+  int bi = kIntMax;
+  for (int v = (int)threadIdx.x * VEC; v < V; v += kCluThreads * VEC) {
+    const uint4 q = load_logits<T>(tp, v, V, vec_ok);
+#pragma unroll
+    for (int k = 0; k < VEC; ++k) {
+      const float z = logit_at<T>(q, k);
+      if (v + k < V && (z > bm || (z == bm && v + k < bi))) {
+        bm = z;
+        bi = v + k;
+      }
+    }
+  }
+  // (value, index) as one 64-bit key: the value's bits in increasing order
+  // (-0 taken as +0, so that equal values tie), then the complemented index
+  uint32_t ub = __float_as_uint(bm + 0.0f);
+  ub = (ub & 0x80000000u) ? ~ub : (ub | 0x80000000u);
+  const uint32_t um = __reduce_max_sync(kFull, ub);
+  const uint32_t ui = __reduce_max_sync(kFull, ub == um ? ~(uint32_t)bi : 0u);
+  if ((threadIdx.x & 31) == 0) atomicMax(s_am, ((unsigned long long)um << 32) | ui);
+  __syncthreads();
+  return (int)~(uint32_t)(*s_am);
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bound_kernel(const StreamArgs a) {
   constexpr int VEC = Elem<T>::kVec;
@@ -1751,6 +1788,8 @@ __global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bou
   __shared__ float s_rk[kCluCtas];       // rank 0: each CTA's (key, group, token)
   __shared__ int s_rg[kCluCtas];
   __shared__ int s_rt[kCluCtas];
+  __shared__ int s_fb;                   // rank 0: the row's token, or -1 for the argmax fallback
+  __shared__ unsigned long long s_am;    // rank 0: row_argmax_cta's reduction
   cg::cluster_group cl = cg::this_cluster();
   const int cr = (int)cl.block_rank();
   const int lane = threadIdx.x & 31;
@@ -1905,21 +1944,27 @@ __global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bou
       }
     }
     cl.sync();                             // every CTA's result is in rank 0
-    if (cr == 0 && threadIdx.x == 0) {
-      float k = pos_inf();
-      int g = kIntMax, tok = -1;
+    if (cr == 0) {
+      if (threadIdx.x == 0) {
+        float k = pos_inf();
+        int g = kIntMax, tok = -1;
 #pragma unroll 1
-      for (int c = 0; c < kCluCtas; ++c) {
-        const float kc = s_rk[c];
-        const int gc = s_rg[c];
-        if (kc < k || (kc == k && gc < g)) {
-          k = kc;
-          g = gc;
-          tok = s_rt[c];
+        for (int c = 0; c < kCluCtas; ++c) {
+          const float kc = s_rk[c];
+          const int gc = s_rg[c];
+          if (kc < k || (kc == k && gc < g)) {
+            k = kc;
+            g = gc;
+            tok = s_rt[c];
+          }
         }
+        s_fb = (g == kIntMax || tok < 0) ? -1 : tok;
+        s_am = 0ull;
       }
-      if (g == kIntMax || tok < 0) tok = __ldcg(W.row_targmax + r);   // empty residual: the argmax
-      a.out_tokens[(size_t)b * a.Ko + pos] = tok;
+      __syncthreads();
+      int tok = s_fb;
+      if (tok < 0) tok = row_argmax_cta<T>(tp, a.V, vec_ok, &s_am);   // empty residual: the argmax
+      if (threadIdx.x == 0) a.out_tokens[(size_t)b * a.Ko + pos] = tok;
     }
   }
   // (the per-sequence slots need no clearing: every call writes all of them)

@@ -133,3 +133,33 @@ def test_rows_at_16_byte_offsets(cmsd, dtype):
         o = cmsd.confidence_verify(d, t, tok, p=p, seed=w.seed, iteration=it)
         g = {k: v.cpu().numpy() for k, v in o.items() if v is not None}
         compare(w, g, oracle_fused(w, p, iteration=it))
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_decisions_without_signal_outputs(cmsd, dtype):
+    # Without the per-position signals the pass does not re-read the vectors
+    # holding the maxima. Each lane's vector start then stands in for the
+    # argmax index in the merges. Drafter rows whose maximum value repeats
+    # check that the second-largest logit still sees the repeat (margin 0):
+    # - in the same 16-byte vector;
+    # - 64 entries on (another lane);
+    # - half a row on (another warp).
+    rng = np.random.default_rng(9)
+    B, K, V = 8, 6, 40000
+    d, t, tok = _synthetic(rng, B, K, V, sd=1.5, noise=1.0)
+    for b in range(B):
+        for i in range(K):
+            j = int(np.argmax(d[b, i]))
+            for off in ((1, 64, V // 2), (1,), (64,), (V // 2,), ())[(b + i) % 5]:
+                d[b, i, (j + off) % V] = d[b, i, j]
+    w = _wl(d, t, tok, dtype)
+    p = cmsd.params(K, "sampled", beta_rank=0, tau_base=0.0)
+    dd = cmsd.to_device_logits(w.draft, w.dtype)
+    tt = cmsd.to_device_logits(w.target, w.dtype)
+    tk = torch.from_numpy(w.tokens).cuda()
+    for it in range(3):
+        full = gpu_fused(cmsd, torch, w, p, iteration=it)
+        compare(w, full, oracle_fused(w, p, iteration=it))
+        o = cmsd.confidence_verify(dd, tt, tk, p=p, seed=w.seed, iteration=it, signals=False)
+        for k in ("n_accept", "out_tokens", "k_next"):
+            assert np.array_equal(o[k].cpu().numpy(), full[k]), k
