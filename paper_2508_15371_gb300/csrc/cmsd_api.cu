@@ -278,6 +278,7 @@ int launch(int dtype, int mode, bool sampled, StreamArgs& a, void* ws, size_t ws
       // drain: return the queue counters to zero so the workspace stays usable
       cudaMemsetAsync(a.ws.rec_count, 0, sizeof(int), s);
       cudaMemsetAsync(a.ws.res_cta_done, 0, sizeof(int), s);
+      if (bound) cudaMemsetAsync(a.ws.rec, 0, (size_t)a.B * sizeof(int4), s);   // the released record words
       return cuda_fail(e);
     }
   }

@@ -603,12 +603,21 @@ __device__ __forceinline__ int next_k(const StreamArgs& a, unsigned long long cs
   return k < a.k_min ? a.k_min : k;
 }
 
+// The word of sequence b's record that the bounded residual draw polls:
+// valid bit | kind << 1 | rejected position << 3.
+__device__ __forceinline__ unsigned* rec_word(const Workspace& W, int b) {
+  return reinterpret_cast<unsigned*>(W.rec + b) + 3;
+}
+
 // Queue the sequence's second-pass record, if it needs one; or, for the
-// bounded residual draw, write it (kSeqNone included) at the sequence's own
-// slot, with no atomic round trip at the end of the epilogue.
+// bounded residual draw, release it (kSeqNone included) at the sequence's own
+// slot: one word that the draw polls, written after every other write of the
+// epilogue (the caller's warp has synchronised) and, through the row
+// counters, of the sequence's rows.
 __device__ __forceinline__ void publish(const StreamArgs& a, int b, int kind, int pos) {
   if (a.rec_by_seq) {
-    a.ws.rec[b] = make_int4(b, pos, kind, 0);
+    const unsigned w = 1u | ((unsigned)kind << 1) | ((unsigned)pos << 3);
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(rec_word(a.ws, b)), "r"(w) : "memory");
     return;
   }
   if (kind == kSeqNone) return;
@@ -655,6 +664,7 @@ __device__ __forceinline__ void seq_epilogue_packed(const StreamArgs& a, int b, 
   }
   if (MODE != kModeConf) {
     write_outputs<MODE, SAMPLED>(a, b, kb, n, lane, tok, (bits >> lane) & 1u);
+    if (PH2) __syncwarp();                 // the lanes' writes precede lane 0's release
     if (PH2 && lane == 0) publish(a, b, seq_kind<MODE, SAMPLED>(a, n, kb), n);
   }
 }
@@ -694,6 +704,7 @@ __device__ __forceinline__ void seq_epilogue_loads(const StreamArgs& a, int b, i
     if (lane == 0) a.n_accept[b] = n;
   }
   if (lane == 0) W.seq_done[b] = 0;
+  if (MODE != kModeConf && PH2) __syncwarp();   // the lanes' writes precede lane 0's release
   if (MODE != kModeConf && PH2 && lane == 0) publish(a, b, seq_kind<MODE, SAMPLED>(a, n, kb), n);
 }
 
@@ -1743,6 +1754,26 @@ __device__ __forceinline__ float group_key(uint4 qt, uint4 qd, const RowStat& st
   return (ok && acc > 0.f) ? expo_u(u) / acc : pos_inf();
 }
 
+// Sequence b's record word, once the streaming kernel's epilogue has released
+// it: polled with acquire loads, giving up after one second (error bit 2 set,
+// and 0 returned, which reads as no record).
+__device__ __forceinline__ unsigned poll_record(const unsigned* p, unsigned* err) {
+  unsigned long long t0;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  for (;;) {
+    unsigned w;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(w) : "l"(p) : "memory");
+    if (w & 1u) return w;
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    if (t - t0 > 1000000000ull) {
+      atomicOr(err, 4u);
+      return 0u;
+    }
+    __nanosleep(32);
+  }
+}
+
 // The verifier row's argmax (the lowest index of its largest logit), by the
 // whole CTA from global memory: the token of a row whose residual is empty.
 // *s_am holds 0 on entry (reset behind a barrier).
@@ -1788,6 +1819,7 @@ __global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bou
   __shared__ float s_rk[kCluCtas];       // rank 0: each CTA's (key, group, token)
   __shared__ int s_rg[kCluCtas];
   __shared__ int s_rt[kCluCtas];
+  __shared__ unsigned s_word;            // the sequence's record word
   __shared__ int s_fb;                   // rank 0: the row's token, or -1 for the argmax fallback
   __shared__ unsigned long long s_am;    // rank 0: row_argmax_cta's reduction
   cg::cluster_group cl = cg::this_cluster();
@@ -1808,17 +1840,30 @@ __global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bou
   const uint32_t cw_grp = iter_word(a.iteration, kPurposeGroup);
   const uint32_t cw_ent = iter_word(a.iteration, kPurposeResidual);
   const int ncl = (int)gridDim.x / kCluCtas;
-  // everything below reads what the streaming kernel wrote: every sequence's
-  // record at its own slot (rec_by_seq)
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // No griddepcontrol.wait here: a sequence's draw starts as soon as its
+  // epilogue has released the record word (every read below follows that
+  // acquire), while the streaming kernel may still be finishing other
+  // sequences.  Its CTAs have all started (they trigger this launch at their
+  // top), so it completes whatever this kernel does.
   const Workspace& W = a.ws;
   // Two cluster barriers per row: after the probes (K1) and after the
   // results.  A slot written before one barrier is read only between it and
   // the next, so no row overwrites what the previous row still reads.
   for (int rr = (int)blockIdx.x / kCluCtas; rr < a.B; rr += ncl) {   // sequence rr, the same for the cluster
-    const int4 rec = __ldcg(W.rec + rr);
-    if (rec.z != kSeqResidual) continue;   // no residual draw for this sequence in this call
-    const int b = rec.x, pos = rec.y;
+    if (threadIdx.x == 0) s_word = poll_record(rec_word(W, rr), W.err);
+    __syncthreads();
+    const unsigned word = s_word;
+    if ((int)((word >> 1) & 3u) != kSeqResidual) {
+      // No residual draw for this sequence in this call: clear the word once
+      // every CTA of the cluster has read it.  The same two cluster barriers
+      // as a draw, so that CTAs that disagree (one poll timed out) still
+      // meet at every barrier.
+      cl.sync();
+      cl.sync();
+      if (cr == 0 && threadIdx.x == 0) *rec_word(W, rr) = 0u;
+      continue;
+    }
+    const int b = rr, pos = (int)(word >> 3);
     const int r = b * a.K + pos;
     const T* tp = (const T*)a.target + (size_t)r * (size_t)a.V;     // no bonus row: Kt == K
     const T* dp = (const T*)a.draft + (size_t)r * (size_t)a.V;
@@ -1964,10 +2009,15 @@ __global__ void __launch_bounds__(kCluThreads, CMSD_CLU_MIN_BLOCKS) resample_bou
       __syncthreads();
       int tok = s_fb;
       if (tok < 0) tok = row_argmax_cta<T>(tp, a.V, vec_ok, &s_am);   // empty residual: the argmax
-      if (threadIdx.x == 0) a.out_tokens[(size_t)b * a.Ko + pos] = tok;
+      if (threadIdx.x == 0) {
+        a.out_tokens[(size_t)b * a.Ko + pos] = tok;
+        *rec_word(W, rr) = 0u;             // every CTA of the cluster has read it (the barrier above)
+      }
     }
   }
-  // (the per-sequence slots need no clearing: every call writes all of them)
+  // this grid completes only after the streaming grid (whatever comes next on
+  // the stream then sees both)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 // ---------------------------------------------------------------------------
