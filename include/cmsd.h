@@ -127,10 +127,22 @@ int cmsd_params_preset(cmsd_params* p, int K, int rule, int preset);
 size_t cmsd_workspace_bytes(int B, int K, int V);
 int cmsd_workspace_init(void* ws, size_t ws_bytes, void* stream);
 
-/* Device-detected input errors since the last init/read (bit 0: drafted token
- * out of range, bit 1: k_row out of range); clears them.  Synchronises
- * `stream`. */
+/* Device-detected errors since the last init/read (bit 0: drafted token out
+ * of range, bit 1: k_row out of range, bit 2: the residual draw gave up after
+ * waiting one second for a sequence's record, whose correction token then
+ * stays -1); clears them.  Synchronises `stream`. */
 int cmsd_workspace_errors(void* ws, size_t ws_bytes, void* stream, uint32_t* flags_out);
+
+/* Test support, no counterpart in the paper: launches the sampled rule's
+ * residual draw by group bounds alone, after clearing the per-sequence record
+ * words that the streaming pass would release.  No record ever appears, so
+ * every sequence's bounded wait runs out (about one second) and sets bit 2
+ * of the error word; nothing else is written (out_tokens, int32 [B][K],
+ * stays as it was).  Arguments as for cmsd_confidence_verify.  Returns
+ * CMSD_EDTYPE, launching nothing, where the bounded draw does not take rows
+ * of V entries. */
+int cmsd_test_record_wait_timeout(const void* draft_logits, const void* target_logits, int B, int K, int V,
+                                  int dtype, int32_t* out_tokens, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * Confidence pass (Sec. III.B(1) and (b)) over drafter logits.

@@ -60,6 +60,7 @@ _SIGS = {
     "cmsd_workspace_bytes": (_c_sz, [_c_int, _c_int, _c_int]),
     "cmsd_workspace_init": (_c_int, [_vp, _c_sz, _vp]),
     "cmsd_workspace_errors": (_c_int, [_vp, _c_sz, _vp, ctypes.POINTER(ctypes.c_uint32)]),
+    "cmsd_test_record_wait_timeout": (_c_int, [_vp, _vp, _c_int, _c_int, _c_int, _c_int, _vp, _vp, _c_sz, _vp]),
     "cmsd_confidence": (_c_int, [_vp, _c_int, _c_int, _c_int, _c_int, _vp, _vp,
                                  _vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_sz, _vp]),
     "cmsd_verify": (_c_int, [_vp, _vp, _vp, _vp, _c_int, _c_int, _c_int, _c_int, _vp,

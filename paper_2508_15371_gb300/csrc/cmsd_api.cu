@@ -447,6 +447,39 @@ int cmsd_workspace_errors(void* ws, size_t ws_bytes, void* stream, uint32_t* fla
   return CMSD_OK;
 }
 
+int cmsd_test_record_wait_timeout(const void* draft_logits, const void* target_logits, int B, int K, int V,
+                                  int dtype, int32_t* out_tokens, void* ws, size_t ws_bytes, void* stream) {
+  int rc = check_sizes(B, K, V, dtype, nullptr);
+  if (rc) return rc;
+  if (B == 0 || K == 0) return CMSD_OK;
+  if (!draft_logits || !target_logits || !out_tokens) return CMSD_EINVAL;
+  if (!aligned16(draft_logits) || !aligned16(target_logits)) return CMSD_EALIGN;
+  if (!resample_bound_fits(dtype, V)) return CMSD_EDTYPE;
+  int wmax = 0;
+  rc = wmax_warps(&wmax);
+  if (rc) return rc;
+  const Layout L = make_layout(B, K, wmax);
+  if (!ws || ws_bytes < L.total) return CMSD_ENOWS;
+  int sms = 0;
+  rc = device_sms(&sms);
+  if (rc) return rc;
+  StreamArgs a = blank_args();
+  fill_sizes(a, B, K, V);
+  a.draft = draft_logits;
+  a.target = target_logits;
+  a.out_tokens = out_tokens;
+  a.Kt = a.Ko = K;
+  a.rec_by_seq = 1;
+  a.ws = carve(ws, L);
+  cudaStream_t s = (cudaStream_t)stream;
+  // no record is released: every sequence's wait runs out
+  cudaError_t e = cudaMemsetAsync(a.ws.rec, 0, (size_t)B * sizeof(int4), s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  const int nclu = B < 2 * sms ? B : 2 * sms;
+  e = dtype == CMSD_F32 ? launch_resample_bound_f32(a, nclu, s) : launch_resample_bound_bf16(a, nclu, s);
+  return e == cudaSuccess ? CMSD_OK : cuda_fail(e);
+}
+
 int cmsd_confidence(const void* draft_logits, int B, int K, int V, int dtype, const int32_t* k_row,
                     const cmsd_params* p, float* H, float* margin, int32_t* argmax, float* conf,
                     float* lse, int32_t* k_next, void* ws, size_t ws_bytes, void* stream) {

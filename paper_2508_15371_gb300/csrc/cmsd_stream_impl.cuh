@@ -1755,18 +1755,19 @@ __device__ __forceinline__ float group_key(uint4 qt, uint4 qd, const RowStat& st
 }
 
 // Sequence b's record word, once the streaming kernel's epilogue has released
-// it: polled with acquire loads, giving up after one second (error bit 2 set,
-// and 0 returned, which reads as no record).
+// it: polled with acquire loads, giving up after one second of globaltimer or
+// 2^22 polls, whichever comes first (error bit 2 set, and 0 returned, which
+// reads as no record).
 __device__ __forceinline__ unsigned poll_record(const unsigned* p, unsigned* err) {
   unsigned long long t0;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
-  for (;;) {
+  for (unsigned n = 0;; ++n) {
     unsigned w;
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(w) : "l"(p) : "memory");
     if (w & 1u) return w;
     unsigned long long t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    if (t - t0 > 1000000000ull) {
+    if (t - t0 > 1000000000ull || n >= (1u << 22)) {
       atomicOr(err, 4u);
       return 0u;
     }

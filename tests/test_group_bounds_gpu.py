@@ -163,3 +163,29 @@ def test_decisions_without_signal_outputs(cmsd, dtype):
         o = cmsd.confidence_verify(dd, tt, tk, p=p, seed=w.seed, iteration=it, signals=False)
         for k in ("n_accept", "out_tokens", "k_next"):
             assert np.array_equal(o[k].cpu().numpy(), full[k]), k
+
+
+def test_record_wait_runs_out(cmsd):
+    # The draw launched alone, with no streaming pass to release the records:
+    # - each sequence's bounded wait gives up after about a second;
+    # - the draw sets error bit 2 and writes no token;
+    # - the context and the workspace then serve an ordinary call.
+    import time
+    rng = np.random.default_rng(10)
+    w = _wl(*_synthetic(rng, 4, 3, 4096, sd=1.0, noise=1.0), "bf16")
+    d = cmsd.to_device_logits(w.draft, w.dtype)
+    t = cmsd.to_device_logits(w.target, w.dtype)
+    ws = cmsd.workspace(w.B, w.K, w.V)
+    out = torch.full((w.B, w.K), 7, dtype=torch.int32, device="cuda")
+    cmsd.workspace_errors(ws)
+    t0 = time.perf_counter()
+    rc = cmsd.lib().cmsd_test_record_wait_timeout(cmsd._ptr(d), cmsd._ptr(t), w.B, w.K, w.V, cmsd.BF16,
+                                                  cmsd._ptr(out), cmsd._ptr(ws), ws.numel(), cmsd._stream())
+    assert rc == cmsd.OK
+    torch.cuda.synchronize()
+    assert 0.5 < time.perf_counter() - t0 < 60
+    assert cmsd.workspace_errors(ws) & 4
+    assert bool((out == 7).all().item())
+    p = cmsd.params(w.K, "sampled", beta_rank=0, tau_base=-1.0)
+    compare(w, gpu_fused(cmsd, torch, w, p, iteration=1), oracle_fused(w, p, iteration=1))
+    assert cmsd.workspace_errors(ws) == 0
